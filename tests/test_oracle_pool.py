@@ -1,0 +1,168 @@
+"""Pins for the reference block pool: the published generator values, the
+shuffle computed by hand from them, and invariants that a wrong refcount,
+a missing copy-on-write or a wrong free order would break."""
+import random
+
+import pytest
+
+from oracle import pool as P
+from conftest import read_golden
+
+MASK = (1 << 64) - 1
+
+
+def test_splitmix64_published_values():
+    want = [int(x[0], 16) for x in read_golden("splitmix64_seed0.txt")]
+    gen = P.splitmix64(0)
+    assert [next(gen) for _ in want] == want
+
+
+def test_free_list_shuffle_by_hand():
+    # Fisher-Yates on [0,1,2] with the published seed-0 outputs x1, x2:
+    # i=2 swaps with x1 % 3, then i=1 swaps with x2 % 2.
+    x1, x2, _ = [int(x[0], 16) for x in read_golden("splitmix64_seed0.txt")]
+    a = [0, 1, 2]
+    j = x1 % 3
+    a[2], a[j] = a[j], a[2]
+    j = x2 % 2
+    a[1], a[j] = a[j], a[1]
+    assert P.initial_free_list(3, 0) == a
+
+
+@pytest.mark.parametrize("n,seed", [(1, 0), (2, 5), (64, 0), (1000, 123)])
+def test_free_list_is_a_permutation(n, seed):
+    fl = P.initial_free_list(n, seed)
+    assert sorted(fl) == list(range(n))
+
+
+def _check_invariants(pool):
+    live = pool.live()
+    # every reference is held by exactly one table entry of a live sequence
+    counts = [0] * pool.n_blocks
+    for i in live:
+        s = pool.seqs[i]
+        assert len(s.table) == -(-s.length // pool.page)
+        for b in s.table:
+            counts[b] += 1
+    assert counts == pool.ref
+    # conservation: free pages are exactly the unreferenced ones, each once
+    assert len(set(pool.free)) == len(pool.free)
+    assert sorted(pool.free) == [b for b in range(pool.n_blocks) if pool.ref[b] == 0]
+    assert len(pool.free) + sum(1 for r in pool.ref if r > 0) == pool.n_blocks
+
+
+def test_random_operation_sequences_keep_invariants_and_content():
+    r = random.Random(42)
+    for trial in range(30):
+        pool = P.RefPool(n_blocks=r.choice([24, 48, 96]), seed=trial, track_content=True)
+        history = {}   # seq -> list of labels it must read back
+        m = pool.create()
+        history[m] = []
+        for step in range(60):
+            live = pool.live()
+            op = r.random()
+            try:
+                if op < 0.45 and live:
+                    ids = r.sample(live, r.randint(1, min(3, len(live))))
+                    n = r.choice([0, 1, 1, 2, 5, 16, 17, 33])
+                    labels = [[(i, len(history[i]) + t, trial) for t in range(n)] for i in ids]
+                    pool.append(ids, n, labels)
+                    for i, lab in zip(ids, labels):
+                        history[i] += lab
+                elif op < 0.65 and live:
+                    parent = r.choice(live)
+                    for c in pool.fork(parent, r.randint(1, 4)):
+                        history[c] = list(history[parent])
+                elif op < 0.85 and len(live) > 1:
+                    pool.release(r.choice(live))
+                else:
+                    c = pool.create()
+                    history[c] = []
+            except P.OutOfBlocks:
+                pass
+            _check_invariants(pool)
+            for i in pool.live():
+                assert pool.read(i) == history[i]
+
+
+def test_fork_then_release_restores_refcounts_and_free_list():
+    pool = P.RefPool(n_blocks=64, seed=3)
+    m = pool.create()
+    pool.append([m], 40)
+    before = (list(pool.ref), list(pool.free))
+    aux = pool.fork(m, 4)
+    assert all(pool.ref[b] == 5 for b in pool.seqs[m].table)
+    for a in aux:
+        pool.release(a)
+    assert (list(pool.ref), list(pool.free)) == before
+
+
+def test_copy_on_write_first_appender_copies_last_holder_writes_in_place():
+    pool = P.RefPool(n_blocks=32, seed=1)
+    m = pool.create()
+    pool.append([m], 20)              # pages: one full, one with 4 rows
+    partial = pool.seqs[m].table[1]
+    aux = pool.fork(m, 2)
+    ev = pool.append([aux[0]], 1)     # shared partial page -> copy 4 rows
+    assert len(ev) == 1 and ev[0][0] == partial and ev[0][2] == 4
+    ev = pool.append([m], 1)          # still shared by m and aux[1] -> copy
+    assert len(ev) == 1 and ev[0][0] == partial
+    assert pool.ref[partial] == 1     # only aux[1] holds it now
+    ev = pool.append([aux[1]], 1)     # last holder writes in place
+    assert ev == [] and pool.seqs[aux[1]].table[1] == partial
+    # the full first page is never copied
+    assert pool.seqs[aux[0]].table[0] == pool.seqs[m].table[0] == pool.seqs[aux[1]].table[0]
+
+
+def test_append_at_page_boundary_allocates_without_copy():
+    pool = P.RefPool(n_blocks=16, seed=2)
+    m = pool.create()
+    pool.append([m], 32)
+    aux = pool.fork(m, 1)
+    free_before = len(pool.free)
+    assert pool.append(aux, 1) == []
+    assert len(pool.free) == free_before - 1
+    assert pool.seqs[aux[0]].table[:2] == pool.seqs[m].table
+
+
+def test_allocation_follows_the_fifo_and_release_refills_its_tail():
+    pool = P.RefPool(n_blocks=8, seed=9)
+    order = P.initial_free_list(8, 9)
+    a = pool.create()
+    pool.append([a], 48)                       # three pages: the FIFO head
+    assert pool.seqs[a].table == order[:3]
+    pool.release(a)
+    assert list(pool.free) == order[3:] + order[:3]
+
+
+def test_out_of_blocks_changes_nothing():
+    pool = P.RefPool(n_blocks=4, seed=0)
+    a = pool.create()
+    b = pool.create()
+    pool.append([a], 40)                       # 3 pages
+    snap = (list(pool.ref), list(pool.free), list(pool.seqs[a].table), pool.seqs[a].length)
+    with pytest.raises(P.OutOfBlocks):
+        pool.append([b, a], 16)                # needs 1 + 1 > 1 free
+    assert snap == (list(pool.ref), list(pool.free), list(pool.seqs[a].table), pool.seqs[a].length)
+    assert pool.seqs[b].length == 0
+
+
+def test_out_of_slots_changes_nothing():
+    pool = P.RefPool(n_blocks=8, seed=0, max_seqs=3)
+    a = pool.create()
+    pool.append([a], 5)
+    snap = list(pool.ref)
+    with pytest.raises(P.OutOfSlots):
+        pool.fork(a, 3)
+    assert pool.ref == snap and len(pool.live()) == 1
+
+
+def test_merge_is_an_append_to_main():
+    p1 = P.RefPool(n_blocks=32, seed=4)
+    p2 = P.RefPool(n_blocks=32, seed=4)
+    for p in (p1, p2):
+        m = p.create()
+        p.append([m], 37)
+    p1.merge(0, 50)
+    p2.append([0], 50)
+    assert p1.seqs[0].table == p2.seqs[0].table and list(p1.free) == list(p2.free)
