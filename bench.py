@@ -1,0 +1,374 @@
+"""Fork-group decode benchmark: branch-steps/s and achieved HBM bandwidth.
+
+Workload (default): the long-trajectory agent -- 4 independent fork groups,
+each a 131072-token shared prefix with 1 main + 4 auxiliary branches holding
+suffixes of up to 2048 tokens; 64 query / 8 KV heads, head_dim 128, 32
+layers, bf16 KV, fp32 outputs.  One step = every branch appends one KV row
+(all layers) and decodes one query (all layers): 20 branch-steps, about
+71 GB of algorithmic KV reads, well beyond the 129 MB L2.
+
+Multi-GPU: fork groups are independent, so N ranks run N replicas with no
+data-path collective (weak scaling); the timing takes the max over ranks.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "fork-group decode branch-steps/s and achieved HBM GB/s vs GB300 peak (1 GPU)"
+UNIT = "branch-steps/s"
+PREFIX_CHUNK = 8192
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    if ws <= 1:
+        return 0, 1, 0
+    import torch
+    import torch.distributed as dist
+    rank = int(os.environ["RANK"])
+    local = int(os.environ.get("LOCAL_RANK", rank))
+    torch.cuda.set_device(local)
+    dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return rank, ws, local
+
+
+def _barrier_max(x, ws):
+    if ws <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu):
+        self.gpu = gpu
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) != len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax = float(parts[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def _kernel_hash():
+    h = hashlib.sha256()
+    for f in ("attend.cu", "ptx.cuh", "kernels.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_13667_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def _ncu_traffic(kernel):
+    """dram bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
+            d = json.load(f)
+    except OSError:
+        return None
+    e = d.get(kernel)
+    if not e or e.get("source_hash") != _kernel_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# --------------------------------------------------------------------------- ours
+
+def build_long_workload(w, dev):
+    """Pool with 4 fork groups at full size; returns (pool, branch handles)."""
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import kv_rows
+    pool = st.Pool(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                   head_dim=w.head_dim, n_blocks=w.n_blocks, seed=w.seed, device=dev, **w.limits)
+    shape = lambda n: (w.n_layers, 1, n, w.n_kv_heads, w.head_dim)
+    branches = []
+    for t in range(w.n_tasks):
+        m = pool.seq_create()
+        for c0 in range(0, w.prefix[t], PREFIX_CHUNK):
+            n = min(PREFIX_CHUNK, w.prefix[t] - c0)
+            k, v = kv_rows(w, ("prefix", t, c0), n, device=dev)
+            pool.append_kv([m], k.view(shape(n)), v.view(shape(n)))
+            del k, v
+        br = [m] + pool.fork(m, w.n_aux)
+        for b, (h, s) in enumerate(zip(br, w.suffix[t])):
+            if s:
+                k, v = kv_rows(w, ("suffix", t, b), s, device=dev)
+                pool.append_kv([h], k.view(shape(s)), v.view(shape(s)))
+        branches += br
+    torch.cuda.synchronize(dev)
+    return pool, branches
+
+
+def run_ours(args, rank, ws, local):
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import get, kv_rows, queries
+    w = get(args.config)
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    st.build()
+    pool, br = build_long_workload(w, dev)
+    n_br = len(br)
+    n_steps = args.warmup + args.steps
+    # per-step inputs, resident in HBM before the timed region
+    step_k, step_v, step_q = [], [], []
+    for s in range(n_steps):
+        k, v = kv_rows(w, ("step", s, rank), n_br, device=dev)
+        step_k.append(k.view(w.n_layers, n_br, 1, w.n_kv_heads, w.head_dim))
+        step_v.append(v.view(w.n_layers, n_br, 1, w.n_kv_heads, w.head_dim))
+        step_q.append(queries(w, ("q", s, rank), n_br, device=dev))
+    o = torch.empty((w.n_layers, n_br, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+    lse = torch.empty((w.n_layers, n_br, w.n_q_heads), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(s):
+        pool.append_kv(br, step_k[s], step_v[s])
+        pool.decode_attn(br, step_q[s], o, lse)
+
+    for s in range(args.warmup):
+        step(s)
+    pool.sync()
+    pool.profile_read()  # drop warm-up counts
+    pool.profile_enable(True)
+    clocks = ClockSampler(local)
+    _barrier(ws)
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(args.warmup, n_steps):
+        step(s)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    clk = clocks.stop()
+    _barrier(ws)
+    ms = e0.elapsed_time(e1)
+    pool.sync()
+    stats = pool.profile_read()
+    pool.profile_enable(False)
+    ms_max = _barrier_max(ms, ws)
+
+    # end-to-end through the public API with host buffers: H2D of the step's
+    # q and new K/V rows from pinned memory, D2H of O and LSE, every step
+    e2e_steps = max(2, min(args.steps, 5))
+    hq = [step_q[s % n_steps].cpu().pin_memory() for s in range(e2e_steps)]
+    hk = [step_k[s % n_steps].cpu().pin_memory() for s in range(e2e_steps)]
+    hv = [step_v[s % n_steps].cpu().pin_memory() for s in range(e2e_steps)]
+    ho = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    hl = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    dq, dk, dv = torch.empty_like(step_q[0]), torch.empty_like(step_k[0]), torch.empty_like(step_v[0])
+    _barrier(ws)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for s in range(e2e_steps):
+        dq.copy_(hq[s], non_blocking=True)
+        dk.copy_(hk[s], non_blocking=True)
+        dv.copy_(hv[s], non_blocking=True)
+        pool.append_kv(br, dk, dv)
+        pool.decode_attn(br, dq, o, lse)
+        ho.copy_(o, non_blocking=True)
+        hl.copy_(lse, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    e2e_s = _barrier_max(time.perf_counter() - t0, ws)
+    h2d = hq[0].numel() * 2 + hk[0].numel() * 2 * 2
+    d2h = ho.numel() * 4 + hl.numel() * 4
+
+    res = {}
+    if rank == 0:
+        peaks, src = _peaks()
+        dec = stats["decode_partial"]
+        launches = sum(v["launches"] for v in stats.values())
+        avg_ms = dec["total_ms"] / max(1, dec["launches"])
+        bytes_per_launch = dec["bytes"] / max(1, dec["launches"])
+        achieved = bytes_per_launch / (avg_ms * 1e-3) / 1e9
+        step_bytes = sum(v["bytes"] for v in stats.values()) / args.steps
+        value = ws * n_br * args.steps / (ms_max * 1e-3)
+        res = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "tasks": w.n_tasks, "branches_per_task": w.n_aux + 1,
+                       "prefix_tokens": w.prefix[0], "suffix_tokens": [list(s) for s in w.suffix],
+                       "layers": w.n_layers, "q_heads": w.n_q_heads, "kv_heads": w.n_kv_heads,
+                       "head_dim": w.head_dim, "step": "append 1 KV row + decode, every branch, all layers",
+                       "l2": "inputs larger than L2 (~71 GB of KV per step)",
+                       "parallelism": f"replicas x{ws}"},
+            "hbm_gbs_step": step_bytes / (ms_max / args.steps * 1e-3) / 1e9,
+            "roofline": {"kernel": "decode_partial", "bound": "hbm", "achieved": achieved,
+                         "peak": peaks["hbm_gbs"], "peak_source": src, "unit": "GB/s",
+                         "frac": achieved / peaks["hbm_gbs"], "frac_of_nominal_8tbs": achieved / 8000.0,
+                         "bytes_per_launch": bytes_per_launch, "avg_launch_ms": avg_ms,
+                         "traffic": _ncu_traffic("decode_partial")},
+            "kernels": {k: {"launches": v["launches"], "ms": v["total_ms"]} for k, v in stats.items()
+                        if v["launches"]},
+            "gpu_launches": launches,
+            "clocks": clk,
+            "e2e": {"value": ws * n_br * e2e_steps / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+        }
+    pool.close()
+    return res
+
+
+# --------------------------------------------------------------------------- oracle
+
+def oracle_sample_step(w, dev, layer, task=0):
+    """The float64 oracle over one layer of one fork group (5 branches): a
+    bounded sample of the step.  Returns (seconds of oracle work, branch-steps)."""
+    import torch
+    from oracle import attention as A
+    from workloads import kv_rows, queries
+    ks, vs = [], []
+    for c0 in range(0, w.prefix[task], PREFIX_CHUNK):
+        n = min(PREFIX_CHUNK, w.prefix[task] - c0)
+        k, v = kv_rows(w, ("prefix", task, c0), n, device=dev, layers=[layer])
+        ks.append(k[0].cpu())
+        vs.append(v[0].cpu())
+    pk, pv = torch.cat(ks), torch.cat(vs)
+    q = queries(w, ("q", 0, 0), w.n_aux + 1, device=dev, layers=[layer])[0].cpu()
+    ctx = []
+    for b, s in enumerate(w.suffix[task]):
+        if s:
+            k, v = kv_rows(w, ("suffix", task, b), s, device=dev, layers=[layer])
+            ctx.append((torch.cat([pk, k[0].cpu()]), torch.cat([pv, v[0].cpu()])))
+        else:
+            ctx.append((pk, pv))
+    t0 = time.perf_counter()
+    for b in range(w.n_aux + 1):
+        A.decode(q[b], *ctx[b])
+    dt = time.perf_counter() - t0
+    return dt, (w.n_aux + 1) / w.n_layers
+
+
+def cpu_baseline(w, dev):
+    dt, units = oracle_sample_step(w, dev, layer=0)
+    return {"value": units / dt, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"1 of {w.n_layers} layers of 1 of {w.n_tasks} fork groups (5 branches, "
+                      f"{w.prefix[0]}-token prefix), float64 numpy; {dt:.1f} s"}
+
+
+def run_reference(args, rank, ws, local):
+    import torch
+    from workloads import get
+    w = get(args.config)
+    if rank != 0:
+        return {}
+    dev = torch.device("cuda", local) if torch.cuda.is_available() else torch.device("cpu")
+    for s in range(args.warmup):
+        oracle_sample_step(w, dev, layer=s % w.n_layers)
+    total_dt = total_units = 0.0
+    for s in range(args.steps):
+        dt, units = oracle_sample_step(w, dev, layer=(args.warmup + s) % w.n_layers)
+        total_dt += dt
+        total_units += units
+    value = total_units / total_dt
+    sample = (f"each step: 1 layer of 1 fork group (5 branches, {w.prefix[0]}-token prefix) "
+              f"of the {w.name} workload, float64 numpy oracle")
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_dt / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": w.name, "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    rank, ws, local = _dist()
+    if args.impl == "reference":
+        res = run_reference(args, rank, ws, local)
+    else:
+        res = run_ours(args, rank, ws, local)
+        if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+            import torch
+            from workloads import get
+            res["cpu_baseline"] = cpu_baseline(get(args.config), torch.device("cuda", local))
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

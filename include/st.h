@@ -1,0 +1,191 @@
+/*
+ * st.h -- C ABI of the fork-group attention library (libsecondthought.so).
+ *
+ * Second Thought (arXiv 2608.13667) forks four auxiliary reasoning branches
+ * off an agent's main context when a Thought phase ends (Section 3.2), lets
+ * them decode while the main thread acts and waits (Section 3.1), and merges
+ * their harvested thoughts back after the observation (Section 3.5).  Every
+ * branch receives the same snapshot H_t + R_t, so the KV of that prefix is
+ * shared by all decoding streams (Section 3.3); the branch load is therefore
+ * dominated by cached-prefix reads (Section 4.4, timing and cost analyses).
+ *
+ * This library is the GPU side of that: a paged KV pool with refcounted
+ * copy-on-write block tables (fork, release and the merge's bookkeeping touch
+ * only metadata), a decode kernel that streams every shared prefix page once
+ * for all branches x GQA heads of a fork group, per-branch suffix work, a
+ * log-sum-exp combine, and a causal prefill for the merged thought rows.
+ *
+ * Conventions for every call:
+ *  - Return value: ST_OK or an error code; a failing call changes no state.
+ *    st_last_error() gives a one-line reason for the last failure.
+ *  - Device pointers are plain CUDA device addresses on the pool's device;
+ *    the caller owns them (KV storage, workspace, inputs, outputs).
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls that
+ *    take a stream enqueue work and return without waiting.  All calls on one
+ *    pool must be ordered: use one stream, or order streams with events.
+ *  - A pool is used from one host thread at a time.
+ *  - Sequence handles (st_seq) are (generation << 32 | slot); a handle is
+ *    invalid after st_release, and using it gives ST_ERR_INVALID.
+ *  - bf16 tensors are IEEE bfloat16 bit patterns; fp32 outputs are float.
+ *  - Attention is softmax(q k^T / sqrt(D)) v with the log-sum-exp returned in
+ *    natural log (scale included); query head h reads KV head h / G with
+ *    G = n_q_heads / n_kv_heads.
+ */
+#ifndef ST_H
+#define ST_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define ST_API __attribute__((visibility("default")))
+#else
+#define ST_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ST_OK = 0,
+  ST_ERR_INVALID = 1, /* bad argument, stale handle, or a device-side bounds check fired */
+  ST_ERR_OOM = 2,     /* pool pages or sequence slots exhausted; nothing changed */
+  ST_ERR_STATE = 3,   /* operation not possible in the pool's current mode/state */
+  ST_ERR_CUDA = 4,    /* a CUDA runtime call failed */
+  ST_ERR_TIMEOUT = 5  /* a device-side wait ran past its limit (reported by st_sync) */
+} st_status;
+
+typedef int64_t st_seq;
+typedef struct st_pool st_pool;
+
+/* Pool geometry and capacities.
+ * KV storage layout (bf16, caller-allocated):
+ *   k_pool, v_pool : [n_layers][n_blocks][n_kv_heads][page_size][head_dim]
+ * so one page of one head is page_size*head_dim contiguous bf16 values. */
+typedef struct {
+  int32_t n_layers;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;          /* must divide n_q_heads; G = n_q_heads / n_kv_heads <= 64 */
+  int32_t head_dim;            /* 64 or 128 */
+  int32_t page_size;           /* tokens per page; must be 16 */
+  int32_t max_seqs;            /* live sequences at once (handle slots) */
+  int32_t max_pages;           /* block-table capacity per sequence, in pages */
+  int32_t max_decode_branches; /* branches per st_decode_attn call */
+  int32_t max_splits;          /* partial results per (branch, head, layer) in one decode; 2..32 */
+  int32_t reserved;
+  int64_t n_blocks;            /* physical pages in the pool (each spans all layers and KV heads) */
+  uint64_t seed;               /* seeds the free-list shuffle (splitmix64, Fisher-Yates) */
+} st_config;
+
+/* Bytes of device workspace st_pool_create needs for `cfg` (0 if cfg is invalid).
+ * The workspace holds the device copy of the block tables, the staging area
+ * for per-call plans, the decode partials and the device status word. */
+ST_API size_t st_workspace_bytes(const st_config* cfg);
+
+/* Create a pool over caller-owned storage.
+ * k_pool, v_pool: device bf16 buffers in the layout above, 16-byte aligned.
+ * workspace: device buffer of st_workspace_bytes(cfg) bytes, 256-byte aligned.
+ * device: CUDA device ordinal of the buffers.  device = -1 creates a
+ *   metadata-only pool (k_pool, v_pool and workspace must be NULL): fork,
+ *   append and release then update tables and refcounts without touching any
+ *   GPU, and attention calls return ST_ERR_STATE.
+ * The free list starts as a Fisher-Yates shuffle of [0, n_blocks) driven by
+ * splitmix64(seed): for i = n-1 down to 1, j = next() % (i+1), swap(i, j);
+ * allocation pops the head, freed pages are pushed to the tail.
+ * On success *out owns host memory and a pinned staging buffer; release it
+ * with st_pool_destroy. */
+ST_API st_status st_pool_create(const st_config* cfg, void* k_pool, void* v_pool, void* workspace,
+                                int device, st_pool** out);
+
+/* Free the pool's host state (waits for its outstanding work first).  The
+ * caller's device buffers are not freed. */
+ST_API st_status st_pool_destroy(st_pool* pool);
+
+/* New empty sequence (a main thread).  ST_ERR_OOM when no slot is free. */
+ST_API st_status st_seq_create(st_pool* pool, st_seq* out);
+
+/* Fork (Section 3.2/3.3): create n_aux sequences whose block tables are copies
+ * of `seq`'s, taking one reference on every page; no page is allocated and no
+ * KV byte moves.  All-or-nothing: ST_ERR_OOM if fewer than n_aux slots are
+ * free.  out_aux receives n_aux handles. */
+ST_API st_status st_fork(st_pool* pool, st_seq seq, int n_aux, st_seq* out_aux);
+
+/* Append n_tok KV rows to each of the n_br sequences in br (in that order;
+ * each sequence at most once per call).
+ * k, v: device bf16 [n_layers][n_br][n_tok][n_kv_heads][head_dim].
+ * Row t of branch i lands at logical position len_i + t.  A fresh page is
+ * taken when the position is page-aligned; a shared partial last page
+ * (refcount > 1) is first copied (copy-on-write: new page, rows
+ * [0, len % page) copied for every layer and head, one reference dropped on
+ * the old page).  All-or-nothing: ST_ERR_OOM if the pool lacks the pages the
+ * whole call needs.  On a metadata-only pool k and v must be NULL. */
+ST_API st_status st_append_kv(st_pool* pool, const st_seq* br, int n_br, int n_tok, const void* k,
+                              const void* v, void* stream);
+
+/* Decode attention for one query per branch (Section 3.1: main and branches
+ * decode concurrently).  Branches forked from a common sequence are grouped:
+ * the pages they share are read once for the whole group, each branch's own
+ * pages once for that branch, and the partial results are combined by
+ * log-sum-exp.  The result equals softmax attention over each branch's full
+ * context (every row appended to it or inherited at fork).
+ * q:   device bf16 [n_layers][n_br][n_q_heads][head_dim]
+ * o:   device fp32 [n_layers][n_br][n_q_heads][head_dim]
+ * lse: device fp32 [n_layers][n_br][n_q_heads] (natural log)
+ * Every branch must hold at least one row; n_br <= max_decode_branches;
+ * a sequence may appear once. */
+ST_API st_status st_decode_attn(st_pool* pool, const st_seq* br, int n_br, const void* q, float* o,
+                                float* lse, void* stream);
+
+/* Merge (Section 3.5): append the n_tok harvested thought rows to `main`
+ * (same rules as st_append_kv) and run their causal prefill: thought row i
+ * attends over main's rows [0, L0 + i] inclusive, L0 = main's length before
+ * the call.  q: bf16 [n_layers][n_tok][n_q_heads][head_dim];
+ * k, v: bf16 [n_layers][n_tok][n_kv_heads][head_dim];
+ * o: fp32 [n_layers][n_tok][n_q_heads][head_dim]; lse: fp32 [n_layers][n_tok][n_q_heads].
+ * n_tok = 0 (nothing harvested) is a no-op returning ST_OK.  On a
+ * metadata-only pool all five pointers must be NULL (bookkeeping only). */
+ST_API st_status st_merge(st_pool* pool, st_seq main, int n_tok, const void* q, const void* k,
+                          const void* v, float* o, float* lse, void* stream);
+
+/* Release (Section 3.5: in-flight branches are cancelled and discarded):
+ * drop one reference per table entry in logical order; pages reaching zero
+ * go to the tail of the free list.  The handle becomes invalid. */
+ST_API st_status st_release(st_pool* pool, st_seq seq);
+
+/* Introspection.  st_block_table copies up to `cap` physical page ids of
+ * `seq` (logical order) into out and reports its page and token counts. */
+ST_API st_status st_block_table(st_pool* pool, st_seq seq, int32_t* out, int cap, int* n_pages,
+                                int* n_tokens);
+/* Per-page refcounts, out[n_blocks]. */
+ST_API st_status st_refcounts(st_pool* pool, int32_t* out, int64_t cap);
+/* Free list in FIFO order (head first); *n receives its length. */
+ST_API st_status st_free_list(st_pool* pool, int32_t* out, int64_t cap, int64_t* n);
+
+/* Wait for the stream and report device-side errors raised since the last
+ * st_sync (ST_ERR_TIMEOUT for a wait that ran out, ST_ERR_INVALID for a
+ * failed bounds check); the device status word is then cleared. */
+ST_API st_status st_sync(st_pool* pool, void* stream);
+
+/* Kernel accounting.  Launch counts are always kept; with timing enabled
+ * (st_profile_enable(pool, 1)) each launch is bracketed by CUDA events on
+ * its stream.  st_profile_read synchronises, fills up to cap records and
+ * resets the counters. */
+typedef struct {
+  char name[32];
+  int64_t launches;
+  double total_ms;     /* summed event time (0 when timing was off) */
+  double bytes;        /* algorithmic bytes the launches had to move */
+  double flops;        /* algorithmic floating-point operations */
+} st_kernel_stat;
+ST_API st_status st_profile_enable(st_pool* pool, int enable);
+ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, int* n);
+
+ST_API const char* st_status_str(st_status s);
+ST_API const char* st_last_error(st_pool* pool);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ST_H */

@@ -41,20 +41,22 @@ def decode(q, k_ctx, v_ctx):
     v_ctx  [n, Hkv, D]
     returns o [Hq, D] float64, lse [Hq] float64
     """
-    q, k, v = _f64(q), _f64(k_ctx), _f64(v_ctx)
+    q = _f64(q)
     Hq, D = q.shape
-    n, Hkv, _ = k.shape
+    n, Hkv = k_ctx.shape[0], k_ctx.shape[1]
     if n == 0:
         raise ValueError("decode over an empty context")
     G = Hq // Hkv
     o = np.empty((Hq, D))
     lse = np.empty(Hq)
-    for h in range(Hq):
-        g = h // G
-        s = (k[:, g, :] @ q[h]) / math.sqrt(D)
-        m = s.max()
-        lse[h] = m + math.log(np.exp(s - m).sum())
-        o[h] = np.exp(s - lse[h]) @ v[:, g, :]
+    for g in range(Hkv):
+        # one KV head at a time, widened exactly to float64
+        kg, vg = _f64(k_ctx[:, g, :]), _f64(v_ctx[:, g, :])
+        for h in range(g * G, (g + 1) * G):
+            s = (kg @ q[h]) / math.sqrt(D)
+            m = s.max()
+            lse[h] = m + math.log(np.exp(s - m).sum())
+            o[h] = np.exp(s - lse[h]) @ vg
     return o, lse
 
 
@@ -74,7 +76,7 @@ def merge_prefill(q, k_all, v_all, L0, rows=None):
     returns o [len(rows), Hq, D], lse [len(rows), Hq]
     """
     q = _f64(q)
-    k, v = _f64(k_all), _f64(v_all)
+    k, v = k_all, v_all
     T = q.shape[0]
     rows = range(T) if rows is None else rows
     outs = [decode(q[i], k[: L0 + i + 1], v[: L0 + i + 1]) for i in rows]

@@ -1,0 +1,99 @@
+// Parameter blocks and launchers of the device kernels.
+//
+//   table_update  -- refresh rows of the device block tables from the host's
+//   append_kv     -- copy-on-write page copies + scatter of new K/V rows
+//   attend        -- paged attention partials (decode) / causal prefill (merge)
+//   lse_combine   -- log-sum-exp combine of decode partials
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace st {
+
+constexpr int kPageTokens = 16;
+
+// Device status word codes (mirrors st_status values).
+constexpr int32_t kDevBadIndex = 1;
+constexpr int32_t kDevTimeout = 5;
+
+struct TableRun {
+  int64_t dst;    // slot * max_pages + first entry
+  int32_t count;  // entries
+  int32_t src;    // offset into the values array
+};
+
+struct CowCopy {
+  int32_t src_block;
+  int32_t dst_block;
+  int32_t rows;  // rows [0, rows) of every layer and KV head
+  int32_t pad;
+};
+
+struct AppendBranch {
+  int32_t slot;
+  int32_t start;  // sequence length before this call
+};
+
+struct AppendParams {
+  const __nv_bfloat16* k;  // [L][n_br][n_tok][Hkv][D]
+  const __nv_bfloat16* v;
+  __nv_bfloat16* k_pool;   // [L][n_blocks][Hkv][16][D]
+  __nv_bfloat16* v_pool;
+  const int32_t* table;    // [max_seqs][max_pages]
+  const AppendBranch* branches;
+  const CowCopy* cows;
+  int32_t* status;
+  int64_t n_blocks;
+  int32_t n_cow, n_br, n_tok, L, Hkv, max_pages;
+};
+
+// One unit of decode work: a run of pages of one block table, read for a set
+// of branches ("members") that all hold those pages.
+struct AttnItem {
+  int32_t slot;        // block-table row the page ids come from
+  int32_t page_begin;  // first logical page
+  int32_t n_pages;
+  int32_t n_tokens;    // valid keys in the run (the last page may be partial)
+  int32_t member_base; // index of the first member in the members array
+  int32_t n_members;
+  int32_t split;       // partial slot this item writes
+  int32_t pad;
+};
+
+struct AttnParams {
+  const __nv_bfloat16* q;  // [L][n_rows_q][Hq][D]
+  float* out_o;            // decode: partials [L][n_br][Hq][max_splits][D]; merge: [L][T][Hq][D]
+  float* out_lse;          // decode: [L][n_br][Hq][max_splits];              merge: [L][T][Hq]
+  const int32_t* table;
+  const AttnItem* items;   // decode only
+  const int32_t* members;  // decode only: branch index (in the call) of each member
+  int32_t* status;
+  int64_t n_blocks;
+  float scale_log2;        // log2(e) / sqrt(D)
+  int32_t n_rows_q;        // decode: n_br; merge: T
+  int32_t Hq, Hkv, G, L, max_pages, max_splits;
+  int32_t slot, L0, T;     // merge only: main's slot, length before the append, thought rows
+};
+
+struct CombineParams {
+  const float* part_o;
+  const float* part_lse;
+  float* o;                 // [L][n_br][Hq][D]
+  float* lse;               // [L][n_br][Hq]
+  const int32_t* n_splits;  // [n_br]
+  int32_t n_br, Hq, L, max_splits;
+};
+
+cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int32_t* values,
+                                int n_runs, cudaStream_t s);
+cudaError_t launch_append(const AppendParams& p, int D, cudaStream_t s);
+cudaError_t launch_attend(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
+                          int n_ctas, bool causal, int D, cudaStream_t s);
+cudaError_t launch_combine(const CombineParams& p, int D, cudaStream_t s);
+// CTAs of the attend kernel resident per SM (0 on error).
+int attend_ctas_per_sm(int D, bool causal);
+
+}  // namespace st

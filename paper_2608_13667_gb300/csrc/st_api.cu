@@ -1,0 +1,876 @@
+// C ABI of the fork-group attention library (declared in include/st.h).
+//
+// The host side is authoritative: the block pool (block_pool.cpp) decides
+// every allocation, and each call turns its decision into a small plan that
+// is copied to the device through a pinned staging ring and consumed by the
+// kernels of that call.  Planning for st_decode_attn groups the branches of a
+// call by fork family and finds the pages they share, so the kernels read a
+// shared prefix page once per group (Section 3.3 of the paper).
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/st.h"
+#include "block_pool.h"
+#include "kernels.cuh"
+
+using namespace st;
+
+namespace {
+
+constexpr int kStageSlots = 8;
+constexpr size_t kStageSlotBytes = 2u << 20;  // 2 MiB per plan
+constexpr int kMaxAttnRows = 64;              // stacked query rows per CTA
+
+enum KernelId { kKTable = 0, kKAppend, kKDecode, kKCombine, kKMerge, kNumKernels };
+const char* const kKernelNames[kNumKernels] = {"table_update", "append_kv", "decode_partial",
+                                              "lse_combine", "merge_prefill"};
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct WorkspaceLayout {
+  size_t status = 0, tables = 0, staging = 0, part_o = 0, part_lse = 0, total = 0;
+};
+
+bool config_valid(const st_config* c, std::string* why) {
+  auto bad = [&](const char* m) {
+    if (why) *why = m;
+    return false;
+  };
+  if (!c) return bad("config is NULL");
+  if (c->n_layers < 1) return bad("n_layers must be >= 1");
+  if (c->n_kv_heads < 1 || c->n_q_heads < 1 || c->n_q_heads % c->n_kv_heads != 0)
+    return bad("n_kv_heads must divide n_q_heads");
+  if (c->n_q_heads / c->n_kv_heads > kMaxAttnRows) return bad("n_q_heads / n_kv_heads must be <= 64");
+  if (c->head_dim != 64 && c->head_dim != 128) return bad("head_dim must be 64 or 128");
+  if (c->page_size != kPageTokens) return bad("page_size must be 16");
+  if (c->max_seqs < 1) return bad("max_seqs must be >= 1");
+  if (c->max_pages < 1) return bad("max_pages must be >= 1");
+  if (c->max_decode_branches < 1) return bad("max_decode_branches must be >= 1");
+  if (c->max_splits < 2 || c->max_splits > 32) return bad("max_splits must be in [2, 32]");
+  if (c->n_blocks < 1 || c->n_blocks > (int64_t)INT32_MAX) return bad("n_blocks out of range");
+  if ((int64_t)c->n_layers * c->n_blocks >= (int64_t)INT32_MAX)
+    return bad("n_layers * n_blocks must be < 2^31");
+  if ((int64_t)c->n_kv_heads * kPageTokens > 65535) return bad("too many KV heads");
+  return true;
+}
+
+WorkspaceLayout layout_for(const st_config* c) {
+  WorkspaceLayout w;
+  size_t off = 0;
+  w.status = off;
+  off = align_up(off + 64, 256);
+  w.tables = off;
+  off = align_up(off + (size_t)c->max_seqs * c->max_pages * sizeof(int32_t), 256);
+  w.staging = off;
+  off = align_up(off + (size_t)kStageSlots * kStageSlotBytes, 256);
+  const size_t n_part = (size_t)c->max_decode_branches * c->n_layers * c->n_q_heads * c->max_splits;
+  w.part_o = off;
+  off = align_up(off + n_part * c->head_dim * sizeof(float), 256);
+  w.part_lse = off;
+  off = align_up(off + n_part * sizeof(float), 256);
+  w.total = off;
+  return w;
+}
+
+struct KStat {
+  int64_t launches = 0;
+  double ms = 0, bytes = 0, flops = 0;
+};
+
+struct PendingTiming {
+  int kid;
+  cudaEvent_t e0, e1;
+};
+
+// Plan writer over one staging slot: sub-allocations are 16-byte aligned and
+// addressed by the same offset on the host (pinned) and the device side.
+struct Plan {
+  uint8_t* h = nullptr;
+  uint8_t* d = nullptr;
+  size_t cap = 0, off = 0;
+  template <class T>
+  T* alloc(size_t n, const T** dev) {
+    off = align_up(off, 16);
+    if (off + n * sizeof(T) > cap) return nullptr;
+    T* hp = reinterpret_cast<T*>(h + off);
+    *dev = reinterpret_cast<const T*>(d + off);
+    off += n * sizeof(T);
+    return hp;
+  }
+};
+
+}  // namespace
+
+struct st_pool {
+  st_config cfg{};
+  BlockPool* pool = nullptr;
+  bool meta_only = false;
+  int device = -1;
+  __nv_bfloat16* k_pool = nullptr;
+  __nv_bfloat16* v_pool = nullptr;
+  uint8_t* ws = nullptr;
+  WorkspaceLayout lay;
+  int32_t* d_status = nullptr;
+  int32_t* d_tables = nullptr;
+  float* d_part_o = nullptr;
+  float* d_part_lse = nullptr;
+  CUtensorMap kmap{}, vmap{};
+  int sms = 0, decode_ctas_per_sm = 0;
+  // staging ring
+  uint8_t* h_stage = nullptr;
+  cudaEvent_t stage_ev[kStageSlots] = {};
+  bool stage_used[kStageSlots] = {};
+  int stage_next = 0;
+  // accounting
+  bool timing = false;
+  KStat stats[kNumKernels];
+  std::vector<PendingTiming> pending;
+  std::vector<cudaEvent_t> spare_events;
+  std::string err;
+};
+
+namespace {
+
+st_status fail(st_pool* P, st_status s, const char* fmt, ...) {
+  if (P) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    P->err = buf;
+  }
+  return s;
+}
+
+#define CUDA_TRY(P, call)                                                                     \
+  do {                                                                                        \
+    cudaError_t e_ = (call);                                                                  \
+    if (e_ != cudaSuccess)                                                                    \
+      return fail((P), ST_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_));          \
+  } while (0)
+
+// Makes the pool's device current for the duration of a call.
+struct DeviceGuard {
+  int prev = -1;
+  bool changed = false;
+  explicit DeviceGuard(int dev) {
+    if (dev < 0) return;
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) {
+      if (cudaSetDevice(dev) == cudaSuccess) changed = true;
+    }
+  }
+  ~DeviceGuard() {
+    if (changed) cudaSetDevice(prev);
+  }
+};
+
+bool decode_handle(st_pool* P, st_seq h, int* slot) {
+  const int64_t s = h & 0xffffffffll;
+  const uint32_t gen = (uint32_t)((uint64_t)h >> 32);
+  if (s < 0 || s >= P->pool->max_seqs()) return false;
+  const SeqSlot& ss = P->pool->slot((int)s);
+  if (!ss.live || ss.gen != gen) return false;
+  *slot = (int)s;
+  return true;
+}
+
+st_seq make_handle(st_pool* P, int slot) {
+  return (st_seq)(((uint64_t)P->pool->slot(slot).gen << 32) | (uint32_t)slot);
+}
+
+cudaEvent_t take_event(st_pool* P) {
+  if (!P->spare_events.empty()) {
+    cudaEvent_t e = P->spare_events.back();
+    P->spare_events.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Launch wrapper: counts the launch, adds its algorithmic bytes/flops, and
+// brackets it with events when timing is on.
+template <class F>
+st_status run_kernel(st_pool* P, int kid, double bytes, double flops, cudaStream_t s, F&& launch) {
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (P->timing) {
+    e0 = take_event(P);
+    cudaEventRecord(e0, s);
+  }
+  const cudaError_t e = launch();
+  if (e != cudaSuccess)
+    return fail(P, ST_ERR_CUDA, "%s launch failed: %s", kKernelNames[kid], cudaGetErrorString(e));
+  if (P->timing) {
+    e1 = take_event(P);
+    cudaEventRecord(e1, s);
+    P->pending.push_back({kid, e0, e1});
+  }
+  KStat& k = P->stats[kid];
+  k.launches += 1;
+  k.bytes += bytes;
+  k.flops += flops;
+  return ST_OK;
+}
+
+// Takes the next staging slot, waiting for the work that last used it.
+st_status acquire_plan(st_pool* P, Plan* plan, int* slot_out) {
+  const int i = P->stage_next;
+  P->stage_next = (i + 1) % kStageSlots;
+  if (P->stage_used[i]) CUDA_TRY(P, cudaEventSynchronize(P->stage_ev[i]));
+  plan->h = P->h_stage + (size_t)i * kStageSlotBytes;
+  plan->d = P->ws + P->lay.staging + (size_t)i * kStageSlotBytes;
+  plan->cap = kStageSlotBytes;
+  plan->off = 0;
+  *slot_out = i;
+  return ST_OK;
+}
+
+st_status submit_plan(st_pool* P, const Plan& plan, cudaStream_t s) {
+  if (plan.off) CUDA_TRY(P, cudaMemcpyAsync(plan.d, plan.h, plan.off, cudaMemcpyHostToDevice, s));
+  return ST_OK;
+}
+
+st_status retire_plan(st_pool* P, int slot, cudaStream_t s) {
+  CUDA_TRY(P, cudaEventRecord(P->stage_ev[slot], s));
+  P->stage_used[slot] = true;
+  return ST_OK;
+}
+
+// Refresh the device copy of every block-table range the host changed.
+st_status flush_tables(st_pool* P, cudaStream_t s) {
+  BlockPool& bp = *P->pool;
+  int slot = 0;
+  const int n = bp.max_seqs();
+  while (slot < n) {
+    Plan plan;
+    int ps;
+    bool any = false;
+    for (int i = slot; i < n; ++i)
+      if (bp.slot(i).live && bp.slot(i).dirty_hi > bp.slot(i).dirty_lo) {
+        any = true;
+        break;
+      }
+    if (!any) return ST_OK;
+    st_status st = acquire_plan(P, &plan, &ps);
+    if (st != ST_OK) return st;
+    // runs first (bounded count), then values
+    const int max_runs = 4096;
+    const TableRun* d_runs;
+    TableRun* runs = plan.alloc<TableRun>(max_runs, &d_runs);
+    const size_t vals_cap = (plan.cap - plan.off - 64) / sizeof(int32_t);
+    const int32_t* d_vals;
+    int32_t* vals = plan.alloc<int32_t>(vals_cap, &d_vals);
+    int n_runs = 0;
+    size_t n_vals = 0;
+    for (; slot < n && n_runs < max_runs; ++slot) {
+      SeqSlot& ss = bp.slot_mut(slot);
+      if (!ss.live || ss.dirty_hi <= ss.dirty_lo) continue;
+      const size_t cnt = (size_t)(ss.dirty_hi - ss.dirty_lo);
+      const size_t room = vals_cap - n_vals;
+      if (room == 0) break;
+      const size_t take = std::min(cnt, room);
+      runs[n_runs] = TableRun{(int64_t)slot * bp.max_pages() + ss.dirty_lo, (int32_t)take, (int32_t)n_vals};
+      std::memcpy(vals + n_vals, ss.table.data() + ss.dirty_lo, take * sizeof(int32_t));
+      n_vals += take;
+      ++n_runs;
+      ss.dirty_lo += (int32_t)take;
+      if (ss.dirty_lo < ss.dirty_hi) break;  // slot only partly uploaded: continue it next round
+      ss.dirty_lo = ss.dirty_hi = 0;
+    }
+    st = submit_plan(P, plan, s);
+    if (st != ST_OK) return st;
+    int32_t* tbl = P->d_tables;
+    st = run_kernel(P, kKTable, (double)n_vals * 8 + n_runs * 16, 0, s,
+                    [&] { return launch_table_update(tbl, d_runs, d_vals, n_runs, s); });
+    if (st != ST_OK) return st;
+    st = retire_plan(P, ps, s);
+    if (st != ST_OK) return st;
+  }
+  return ST_OK;
+}
+
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Validates and performs an append (shared by st_append_kv and st_merge).
+st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const void* k, const void* v,
+                    cudaStream_t s) {
+  BlockPool& bp = *P->pool;
+  int64_t need = 0;
+  for (int i = 0; i < n_br; ++i) {
+    if (!bp.fits(slots[i], n_tok))
+      return fail(P, ST_ERR_OOM, "sequence would exceed max_pages (%d)", bp.max_pages());
+    need += bp.pages_needed(slots[i], n_tok);
+  }
+  if (need > bp.free_count())
+    return fail(P, ST_ERR_OOM, "pool has %lld free pages, call needs %lld",
+                (long long)bp.free_count(), (long long)need);
+  std::vector<int32_t> starts(n_br);
+  for (int i = 0; i < n_br; ++i) starts[i] = (int32_t)bp.slot(slots[i]).len;
+  std::vector<CowEvent> cows;
+  bp.append(slots, n_br, n_tok, &cows);
+  if (P->meta_only || n_tok == 0) return ST_OK;
+
+  st_status st = flush_tables(P, s);
+  if (st != ST_OK) return st;
+  Plan plan;
+  int ps;
+  st = acquire_plan(P, &plan, &ps);
+  if (st != ST_OK) return st;
+  const AppendBranch* d_br;
+  AppendBranch* br = plan.alloc<AppendBranch>(n_br, &d_br);
+  const CowCopy* d_cow;
+  CowCopy* cw = plan.alloc<CowCopy>(std::max<size_t>(cows.size(), 1), &d_cow);
+  if (!br || !cw) return fail(P, ST_ERR_INVALID, "append plan does not fit the staging slot");
+  for (int i = 0; i < n_br; ++i) br[i] = AppendBranch{slots[i], starts[i]};
+  for (size_t i = 0; i < cows.size(); ++i)
+    cw[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
+  st = submit_plan(P, plan, s);
+  if (st != ST_OK) return st;
+  const st_config& c = P->cfg;
+  AppendParams ap{};
+  ap.k = static_cast<const __nv_bfloat16*>(k);
+  ap.v = static_cast<const __nv_bfloat16*>(v);
+  ap.k_pool = P->k_pool;
+  ap.v_pool = P->v_pool;
+  ap.table = P->d_tables;
+  ap.branches = d_br;
+  ap.cows = d_cow;
+  ap.status = P->d_status;
+  ap.n_blocks = c.n_blocks;
+  ap.n_cow = (int32_t)cows.size();
+  ap.n_br = n_br;
+  ap.n_tok = n_tok;
+  ap.L = c.n_layers;
+  ap.Hkv = c.n_kv_heads;
+  ap.max_pages = c.max_pages;
+  const double row_bytes = (double)c.n_layers * c.n_kv_heads * c.head_dim * 2 * 2;
+  double cow_rows = 0;
+  for (auto& e : cows) cow_rows += e.rows;
+  const double bytes = row_bytes * ((double)n_br * n_tok * 2 + cow_rows * 2);
+  st = run_kernel(P, kKAppend, bytes, 0, s, [&] { return launch_append(ap, c.head_dim, s); });
+  if (st != ST_OK) return st;
+  return retire_plan(P, ps, s);
+}
+
+// Longest common prefix (in pages) of two block tables.
+int32_t lcp_pages(const std::vector<int32_t>& a, const std::vector<int32_t>& b) {
+  const size_t n = std::min(a.size(), b.size());
+  size_t i = 0;
+  while (i < n && a[i] == b[i]) ++i;
+  return (int32_t)i;
+}
+
+void split_even(int32_t n, int32_t k, int32_t c, int32_t* begin, int32_t* count) {
+  const int32_t base = n / k, rem = n % k;
+  *begin = c * base + std::min(c, rem);
+  *count = base + (c < rem ? 1 : 0);
+}
+
+}  // namespace
+
+extern "C" {
+
+ST_API const char* st_status_str(st_status s) {
+  switch (s) {
+    case ST_OK: return "ok";
+    case ST_ERR_INVALID: return "invalid argument";
+    case ST_ERR_OOM: return "out of pool pages or sequence slots";
+    case ST_ERR_STATE: return "operation not possible in this state";
+    case ST_ERR_CUDA: return "CUDA error";
+    case ST_ERR_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+ST_API const char* st_last_error(st_pool* pool) { return pool ? pool->err.c_str() : ""; }
+
+ST_API size_t st_workspace_bytes(const st_config* cfg) {
+  if (!config_valid(cfg, nullptr)) return 0;
+  return layout_for(cfg).total;
+}
+
+ST_API st_status st_pool_create(const st_config* cfg, void* k_pool, void* v_pool, void* workspace,
+                                int device, st_pool** out) {
+  if (!out) return ST_ERR_INVALID;
+  *out = nullptr;
+  std::string why;
+  if (!config_valid(cfg, &why)) return ST_ERR_INVALID;
+  st_pool* P = new (std::nothrow) st_pool();
+  if (!P) return ST_ERR_OOM;
+  P->cfg = *cfg;
+  P->device = device;
+  P->meta_only = device < 0;
+  if (P->meta_only) {
+    if (k_pool || v_pool || workspace) {
+      delete P;
+      return ST_ERR_INVALID;
+    }
+  } else {
+    if (!k_pool || !v_pool || !workspace || !aligned(k_pool, 16) || !aligned(v_pool, 16) ||
+        !aligned(workspace, 256)) {
+      delete P;
+      return ST_ERR_INVALID;
+    }
+  }
+  P->pool = new (std::nothrow)
+      BlockPool(cfg->n_blocks, cfg->seed, cfg->page_size, cfg->max_seqs, cfg->max_pages);
+  if (!P->pool) {
+    delete P;
+    return ST_ERR_OOM;
+  }
+  if (P->meta_only) {
+    *out = P;
+    return ST_OK;
+  }
+
+  auto bail = [&](st_status s) {
+    st_pool_destroy(P);
+    return s;
+  };
+  DeviceGuard guard(device);
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess || cur != device) return bail(ST_ERR_CUDA);
+  P->k_pool = static_cast<__nv_bfloat16*>(k_pool);
+  P->v_pool = static_cast<__nv_bfloat16*>(v_pool);
+  P->ws = static_cast<uint8_t*>(workspace);
+  P->lay = layout_for(cfg);
+  P->d_status = reinterpret_cast<int32_t*>(P->ws + P->lay.status);
+  P->d_tables = reinterpret_cast<int32_t*>(P->ws + P->lay.tables);
+  P->d_part_o = reinterpret_cast<float*>(P->ws + P->lay.part_o);
+  P->d_part_lse = reinterpret_cast<float*>(P->ws + P->lay.part_lse);
+  if (cudaMemset(P->ws, 0, P->lay.staging) != cudaSuccess) return bail(ST_ERR_CUDA);
+  if (cudaDeviceGetAttribute(&P->sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
+    return bail(ST_ERR_CUDA);
+  P->decode_ctas_per_sm = attend_ctas_per_sm(cfg->head_dim, false);
+  if (P->decode_ctas_per_sm < 1) return bail(ST_ERR_CUDA);
+  if (cudaHostAlloc(reinterpret_cast<void**>(&P->h_stage), (size_t)kStageSlots * kStageSlotBytes,
+                    cudaHostAllocDefault) != cudaSuccess)
+    return bail(ST_ERR_CUDA);
+  for (int i = 0; i < kStageSlots; ++i)
+    if (cudaEventCreateWithFlags(&P->stage_ev[i], cudaEventDisableTiming) != cudaSuccess)
+      return bail(ST_ERR_CUDA);
+
+  // Tensor maps over the pools: dims (64, D/64, 16*Hkv, L*n_blocks), so one
+  // box {64, 1, 16, 1} is 16 tokens x 64 dims of one head = 2 KiB, loaded
+  // with the 128-byte swizzle.
+  PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  cudaDriverEntryPointQueryResult qres;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&encode),
+                                       12000, cudaEnableDefault, &qres) != cudaSuccess ||
+      qres != cudaDriverEntryPointSuccess || !encode)
+    return bail(ST_ERR_CUDA);
+  const int D = cfg->head_dim;
+  cuuint64_t dims[4] = {64, (cuuint64_t)(D / 64), (cuuint64_t)kPageTokens * cfg->n_kv_heads,
+                        (cuuint64_t)cfg->n_layers * (cuuint64_t)cfg->n_blocks};
+  cuuint64_t strides[3] = {128, (cuuint64_t)D * 2, (cuuint64_t)kPageTokens * cfg->n_kv_heads * D * 2};
+  cuuint32_t box[4] = {64, 1, kPageTokens, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  for (int t = 0; t < 2; ++t) {
+    CUresult r = encode(t == 0 ? &P->kmap : &P->vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+                        t == 0 ? k_pool : v_pool, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return bail(ST_ERR_CUDA);
+  }
+  *out = P;
+  return ST_OK;
+}
+
+ST_API st_status st_pool_destroy(st_pool* P) {
+  if (!P) return ST_ERR_INVALID;
+  if (!P->meta_only) {
+    DeviceGuard guard(P->device);
+    for (int i = 0; i < kStageSlots; ++i)
+      if (P->stage_ev[i]) {
+        cudaEventSynchronize(P->stage_ev[i]);
+        cudaEventDestroy(P->stage_ev[i]);
+      }
+    for (auto& t : P->pending) {
+      cudaEventDestroy(t.e0);
+      cudaEventDestroy(t.e1);
+    }
+    for (auto e : P->spare_events) cudaEventDestroy(e);
+    if (P->h_stage) cudaFreeHost(P->h_stage);
+  }
+  delete P->pool;
+  delete P;
+  return ST_OK;
+}
+
+ST_API st_status st_seq_create(st_pool* P, st_seq* out) {
+  if (!P || !out) return ST_ERR_INVALID;
+  const int s = P->pool->create_seq();
+  if (s < 0) return fail(P, ST_ERR_OOM, "no free sequence slot (max_seqs = %d)", P->cfg.max_seqs);
+  *out = make_handle(P, s);
+  return ST_OK;
+}
+
+ST_API st_status st_fork(st_pool* P, st_seq seq, int n_aux, st_seq* out_aux) {
+  if (!P) return ST_ERR_INVALID;
+  int slot;
+  if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+  if (n_aux < 0 || (n_aux > 0 && !out_aux)) return fail(P, ST_ERR_INVALID, "bad n_aux/out_aux");
+  if (n_aux == 0) return ST_OK;
+  std::vector<int> slots(n_aux);
+  if (!P->pool->fork(slot, n_aux, slots.data()))
+    return fail(P, ST_ERR_OOM, "fewer than %d free sequence slots", n_aux);
+  for (int i = 0; i < n_aux; ++i) out_aux[i] = make_handle(P, slots[i]);
+  return ST_OK;
+}
+
+ST_API st_status st_release(st_pool* P, st_seq seq) {
+  if (!P) return ST_ERR_INVALID;
+  int slot;
+  if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+  P->pool->release(slot);
+  return ST_OK;
+}
+
+ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok, const void* k,
+                              const void* v, void* stream) {
+  if (!P) return ST_ERR_INVALID;
+  if (n_br < 0 || n_tok < 0 || (n_br > 0 && !br)) return fail(P, ST_ERR_INVALID, "bad n_br/n_tok");
+  std::vector<int> slots(n_br);
+  for (int i = 0; i < n_br; ++i) {
+    if (!decode_handle(P, br[i], &slots[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+    for (int j = 0; j < i; ++j)
+      if (slots[j] == slots[i]) return fail(P, ST_ERR_INVALID, "sequence listed twice");
+  }
+  if (P->meta_only) {
+    if (k || v) return fail(P, ST_ERR_INVALID, "metadata-only pool takes no KV data");
+  } else if (n_br > 0 && n_tok > 0 && (!k || !v || !aligned(k, 16) || !aligned(v, 16))) {
+    return fail(P, ST_ERR_INVALID, "k and v must be 16-byte aligned device pointers");
+  }
+  if (n_br == 0 || n_tok == 0) return ST_OK;
+  DeviceGuard guard(P->device);
+  return do_append(P, slots.data(), n_br, n_tok, k, v, static_cast<cudaStream_t>(stream));
+}
+
+ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const void* q, float* o,
+                                float* lse, void* stream) {
+  if (!P) return ST_ERR_INVALID;
+  if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
+  if (n_br < 1 || !br) return fail(P, ST_ERR_INVALID, "need at least one branch");
+  if (n_br > P->cfg.max_decode_branches)
+    return fail(P, ST_ERR_INVALID, "n_br %d > max_decode_branches %d", n_br, P->cfg.max_decode_branches);
+  if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
+    return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
+  BlockPool& bp = *P->pool;
+  const st_config& c = P->cfg;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  DeviceGuard guard(P->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  std::vector<int> slots(n_br);
+  for (int i = 0; i < n_br; ++i) {
+    if (!decode_handle(P, br[i], &slots[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+    if (bp.slot(slots[i]).len < 1) return fail(P, ST_ERR_INVALID, "decode over an empty sequence");
+    for (int j = 0; j < i; ++j)
+      if (slots[j] == slots[i]) return fail(P, ST_ERR_INVALID, "sequence listed twice");
+  }
+
+  // ---- group by fork family, find the shared full pages --------------------
+  std::vector<int32_t> shared(n_br, 0);   // pages of branch i read through its group
+  struct Group { std::vector<int> members; int32_t pages; };
+  std::vector<Group> groups;
+  {
+    std::map<int32_t, std::vector<int>> fam;
+    std::vector<int32_t> order;
+    for (int i = 0; i < n_br; ++i) {
+      const int32_t f = bp.slot(slots[i]).family;
+      if (!fam.count(f)) order.push_back(f);
+      fam[f].push_back(i);
+    }
+    const int per_group = std::max(1, kMaxAttnRows / G);
+    for (int32_t f : order) {
+      const std::vector<int>& mem = fam[f];
+      for (size_t b0 = 0; b0 < mem.size(); b0 += per_group) {
+        const size_t b1 = std::min(mem.size(), b0 + per_group);
+        if (b1 - b0 < 2) continue;
+        const SeqSlot& lead = bp.slot(slots[mem[b0]]);
+        int64_t min_len = lead.len;
+        int32_t pages = (int32_t)lead.table.size();
+        for (size_t m = b0 + 1; m < b1; ++m) {
+          const SeqSlot& ss = bp.slot(slots[mem[m]]);
+          pages = std::min(pages, lcp_pages(lead.table, ss.table));
+          min_len = std::min<int64_t>(min_len, ss.len);
+        }
+        pages = std::min<int32_t>(pages, (int32_t)(min_len / kPageTokens));
+        if (pages < 1) continue;
+        Group g;
+        g.members.assign(mem.begin() + b0, mem.begin() + b1);
+        g.pages = pages;
+        for (int i : g.members) shared[i] = pages;
+        groups.push_back(std::move(g));
+      }
+    }
+  }
+
+  // ---- chunking -------------------------------------------------------------
+  int64_t total_pages = 0;
+  for (auto& g : groups) total_pages += g.pages;
+  std::vector<int32_t> own_pages(n_br), own_tokens(n_br);
+  for (int i = 0; i < n_br; ++i) {
+    const SeqSlot& ss = bp.slot(slots[i]);
+    own_pages[i] = (int32_t)ss.table.size() - shared[i];
+    own_tokens[i] = (int32_t)(ss.len - (int64_t)shared[i] * kPageTokens);
+    total_pages += own_pages[i];
+  }
+  const int64_t units = total_pages * c.n_kv_heads * c.n_layers;
+  const int64_t target_ctas = (int64_t)32 * P->sms * P->decode_ctas_per_sm;
+  int64_t chunk = (units + target_ctas - 1) / target_ctas;
+  chunk = std::max<int64_t>(16, (chunk + 3) / 4 * 4);
+  const int max_prefix_chunks = c.max_splits / 2;
+
+  Plan plan;
+  int ps;
+  st_status st = flush_tables(P, s);
+  if (st != ST_OK) return st;
+  st = acquire_plan(P, &plan, &ps);
+  if (st != ST_OK) return st;
+
+  std::vector<AttnItem> items;
+  std::vector<int32_t> members;
+  std::vector<int32_t> n_splits(n_br, 0);
+  double bytes = 0, flops = 0;
+  const double page_bytes = (double)kPageTokens * c.head_dim * 2 * 2;  // K+V, one head
+  for (auto& g : groups) {
+    const int32_t k = (int32_t)std::min<int64_t>(max_prefix_chunks, (g.pages + chunk - 1) / chunk);
+    const int32_t mbase = (int32_t)members.size();
+    for (int i : g.members) members.push_back(i);
+    for (int32_t cidx = 0; cidx < k; ++cidx) {
+      int32_t b, n;
+      split_even(g.pages, k, cidx, &b, &n);
+      items.push_back(AttnItem{slots[g.members[0]], b, n, n * kPageTokens, mbase,
+                               (int32_t)g.members.size(), cidx, 0});
+      bytes += n * page_bytes;
+      flops += 4.0 * g.members.size() * G * n * kPageTokens * c.head_dim;
+    }
+    for (int i : g.members) n_splits[i] = k;
+  }
+  for (int i = 0; i < n_br; ++i) {
+    if (own_pages[i] <= 0) continue;
+    const int32_t room = c.max_splits - n_splits[i];
+    const int32_t k = (int32_t)std::min<int64_t>(room, (own_pages[i] + chunk - 1) / chunk);
+    const int32_t mbase = (int32_t)members.size();
+    members.push_back(i);
+    for (int32_t cidx = 0; cidx < k; ++cidx) {
+      int32_t b, n;
+      split_even(own_pages[i], k, cidx, &b, &n);
+      const int32_t tok = std::min<int32_t>(n * kPageTokens, own_tokens[i] - b * kPageTokens);
+      items.push_back(AttnItem{slots[i], shared[i] + b, n, tok, mbase, 1, n_splits[i] + cidx, 0});
+      bytes += n * page_bytes;
+      flops += 4.0 * G * tok * c.head_dim;
+    }
+    n_splits[i] += k;
+  }
+  // longest runs first so the short ones fill the tail
+  std::stable_sort(items.begin(), items.end(),
+                   [](const AttnItem& a, const AttnItem& b) { return a.n_pages > b.n_pages; });
+  bytes *= (double)c.n_kv_heads * c.n_layers;
+  flops *= (double)c.n_kv_heads * c.n_layers;
+  const double q_bytes = (double)c.n_layers * n_br * c.n_q_heads * c.head_dim * 2;
+  double part_rows = 0;
+  for (auto& it : items) part_rows += (double)it.n_members * G;
+  part_rows *= (double)c.n_kv_heads * c.n_layers;
+  const double part_bytes = part_rows * (c.head_dim + 1) * 4;
+  bytes += q_bytes + part_bytes;
+
+  const AttnItem* d_items;
+  AttnItem* hi = plan.alloc<AttnItem>(items.size(), &d_items);
+  const int32_t* d_members;
+  int32_t* hm = plan.alloc<int32_t>(members.size(), &d_members);
+  const int32_t* d_nsplit;
+  int32_t* hn = plan.alloc<int32_t>(n_br, &d_nsplit);
+  if (!hi || !hm || !hn) return fail(P, ST_ERR_INVALID, "decode plan does not fit the staging slot");
+  std::memcpy(hi, items.data(), items.size() * sizeof(AttnItem));
+  std::memcpy(hm, members.data(), members.size() * sizeof(int32_t));
+  std::memcpy(hn, n_splits.data(), n_br * sizeof(int32_t));
+  st = submit_plan(P, plan, s);
+  if (st != ST_OK) return st;
+
+  AttnParams ap{};
+  ap.q = static_cast<const __nv_bfloat16*>(q);
+  ap.out_o = P->d_part_o;
+  ap.out_lse = P->d_part_lse;
+  ap.table = P->d_tables;
+  ap.items = d_items;
+  ap.members = d_members;
+  ap.status = P->d_status;
+  ap.n_blocks = c.n_blocks;
+  ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c.head_dim));
+  ap.n_rows_q = n_br;
+  ap.Hq = c.n_q_heads;
+  ap.Hkv = c.n_kv_heads;
+  ap.G = G;
+  ap.L = c.n_layers;
+  ap.max_pages = c.max_pages;
+  ap.max_splits = c.max_splits;
+  const int n_items = (int)items.size();
+  st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
+    return launch_attend(P->kmap, P->vmap, ap, n_items, false, c.head_dim, s);
+  });
+  if (st != ST_OK) return st;
+
+  CombineParams cp{};
+  cp.part_o = P->d_part_o;
+  cp.part_lse = P->d_part_lse;
+  cp.o = o;
+  cp.lse = lse;
+  cp.n_splits = d_nsplit;
+  cp.n_br = n_br;
+  cp.Hq = c.n_q_heads;
+  cp.L = c.n_layers;
+  cp.max_splits = c.max_splits;
+  const double cbytes = part_bytes + (double)c.n_layers * n_br * c.n_q_heads * (c.head_dim + 1) * 4;
+  st = run_kernel(P, kKCombine, cbytes, 0, s, [&] { return launch_combine(cp, c.head_dim, s); });
+  if (st != ST_OK) return st;
+  return retire_plan(P, ps, s);
+}
+
+ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, const void* k,
+                          const void* v, float* o, float* lse, void* stream) {
+  if (!P) return ST_ERR_INVALID;
+  int slot;
+  if (!decode_handle(P, main, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+  if (n_tok < 0) return fail(P, ST_ERR_INVALID, "n_tok < 0");
+  if (n_tok == 0) return ST_OK;  // nothing harvested: plain ReAct continues
+  if (P->meta_only) {
+    if (q || k || v || o || lse) return fail(P, ST_ERR_INVALID, "metadata-only pool takes no data");
+    return do_append(P, &slot, 1, n_tok, nullptr, nullptr, nullptr);
+  }
+  if (!q || !k || !v || !o || !lse || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) ||
+      !aligned(o, 16) || !aligned(lse, 4))
+    return fail(P, ST_ERR_INVALID, "q/k/v/o/lse must be aligned device pointers");
+  const st_config& c = P->cfg;
+  const int64_t L0 = P->pool->slot(slot).len;
+  DeviceGuard guard(P->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  st_status st = do_append(P, &slot, 1, n_tok, k, v, s);
+  if (st != ST_OK) return st;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  AttnParams ap{};
+  ap.q = static_cast<const __nv_bfloat16*>(q);
+  ap.out_o = o;
+  ap.out_lse = lse;
+  ap.table = P->d_tables;
+  ap.status = P->d_status;
+  ap.n_blocks = c.n_blocks;
+  ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c.head_dim));
+  ap.n_rows_q = n_tok;
+  ap.Hq = c.n_q_heads;
+  ap.Hkv = c.n_kv_heads;
+  ap.G = G;
+  ap.L = c.n_layers;
+  ap.max_pages = c.max_pages;
+  ap.max_splits = c.max_splits;
+  ap.slot = slot;
+  ap.L0 = (int32_t)L0;
+  ap.T = n_tok;
+  const int64_t rows = (int64_t)n_tok * G;
+  const int n_tiles = (int)((rows + kMaxAttnRows - 1) / kMaxAttnRows);
+  // algorithmic: main's KV once per (layer, head) + Q + O/LSE; flops: causal
+  const double kv_bytes = (double)(L0 + n_tok) * c.n_kv_heads * c.head_dim * 2 * 2 * c.n_layers;
+  const double io_bytes = (double)c.n_layers * n_tok * c.n_q_heads * (c.head_dim * 2 + c.head_dim * 4 + 4);
+  const double keys = (double)n_tok * L0 + (double)n_tok * (n_tok + 1) / 2;
+  const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
+  return run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s, [&] {
+    return launch_attend(P->kmap, P->vmap, ap, n_tiles, true, c.head_dim, s);
+  });
+}
+
+ST_API st_status st_block_table(st_pool* P, st_seq seq, int32_t* out, int cap, int* n_pages,
+                                int* n_tokens) {
+  if (!P) return ST_ERR_INVALID;
+  int slot;
+  if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+  const SeqSlot& ss = P->pool->slot(slot);
+  if (n_pages) *n_pages = (int)ss.table.size();
+  if (n_tokens) *n_tokens = (int)ss.len;
+  if (out && cap > 0) {
+    const int n = std::min<int>(cap, (int)ss.table.size());
+    std::memcpy(out, ss.table.data(), n * sizeof(int32_t));
+  }
+  return ST_OK;
+}
+
+ST_API st_status st_refcounts(st_pool* P, int32_t* out, int64_t cap) {
+  if (!P || !out) return ST_ERR_INVALID;
+  const auto& r = P->pool->refcounts();
+  const int64_t n = std::min<int64_t>(cap, (int64_t)r.size());
+  std::memcpy(out, r.data(), n * sizeof(int32_t));
+  return ST_OK;
+}
+
+ST_API st_status st_free_list(st_pool* P, int32_t* out, int64_t cap, int64_t* n) {
+  if (!P) return ST_ERR_INVALID;
+  std::vector<int32_t> fl;
+  P->pool->free_list(&fl);
+  if (n) *n = (int64_t)fl.size();
+  if (out && cap > 0) std::memcpy(out, fl.data(), std::min<int64_t>(cap, (int64_t)fl.size()) * sizeof(int32_t));
+  return ST_OK;
+}
+
+ST_API st_status st_sync(st_pool* P, void* stream) {
+  if (!P) return ST_ERR_INVALID;
+  if (P->meta_only) return ST_OK;
+  DeviceGuard guard(P->device);
+  CUDA_TRY(P, cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int32_t code = 0;
+  CUDA_TRY(P, cudaMemcpy(&code, P->d_status, sizeof code, cudaMemcpyDeviceToHost));
+  if (code != 0) {
+    CUDA_TRY(P, cudaMemset(P->d_status, 0, sizeof code));
+    if (code == kDevTimeout) return fail(P, ST_ERR_TIMEOUT, "a device-side wait ran past its limit");
+    return fail(P, ST_ERR_INVALID, "a device-side bounds check failed (code %d)", code);
+  }
+  return ST_OK;
+}
+
+ST_API st_status st_profile_enable(st_pool* P, int enable) {
+  if (!P) return ST_ERR_INVALID;
+  P->timing = enable != 0 && !P->meta_only;
+  return ST_OK;
+}
+
+ST_API st_status st_profile_read(st_pool* P, st_kernel_stat* out, int cap, int* n) {
+  if (!P) return ST_ERR_INVALID;
+  if (!P->meta_only) {
+    DeviceGuard guard(P->device);
+    for (auto& t : P->pending) {
+      CUDA_TRY(P, cudaEventSynchronize(t.e1));
+      float ms = 0;
+      CUDA_TRY(P, cudaEventElapsedTime(&ms, t.e0, t.e1));
+      P->stats[t.kid].ms += ms;
+      P->spare_events.push_back(t.e0);
+      P->spare_events.push_back(t.e1);
+    }
+    P->pending.clear();
+  }
+  int k = 0;
+  for (int i = 0; i < kNumKernels; ++i) {
+    if (k < cap && out) {
+      std::memset(&out[k], 0, sizeof(st_kernel_stat));
+      std::snprintf(out[k].name, sizeof out[k].name, "%s", kKernelNames[i]);
+      out[k].launches = P->stats[i].launches;
+      out[k].total_ms = P->stats[i].ms;
+      out[k].bytes = P->stats[i].bytes;
+      out[k].flops = P->stats[i].flops;
+      ++k;
+    }
+    P->stats[i] = KStat{};
+  }
+  if (n) *n = k;
+  return ST_OK;
+}
+
+}  // extern "C"

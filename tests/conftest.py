@@ -23,3 +23,11 @@ def read_golden(name):
             if line:
                 out.append(line.split())
     return out
+
+
+@pytest.fixture(scope="session")
+def stlib():
+    """The built library (compiled here with nvcc if missing or stale)."""
+    import paper_2608_13667_gb300 as stpkg
+    stpkg.build()
+    return stpkg

@@ -1,0 +1,135 @@
+"""Drives the library and the reference pool with the same fork-group
+operations, and materialises any branch's context for the oracle.
+
+Each append draws its rows from workloads.kv_rows under a tag; the harness
+records, per sequence, which (tag, row range) pieces make up its logical
+context (inherited at fork), so the oracle's context for (sequence, layer)
+is rebuilt by re-drawing those pieces -- never read back from the GPU pool.
+"""
+from collections import OrderedDict
+
+import numpy as np
+import torch
+
+import paper_2608_13667_gb300 as stpkg
+from oracle import attention as A
+from oracle import pool as R
+from workloads import kv_rows, queries
+
+# Tolerances (benchmark spec): elementwise |gpu - oracle| <= 2e-3 + 1e-2 |oracle|
+# for O; |gpu - oracle| <= 1e-4 for the log-sum-exp.
+O_ABS, O_REL, LSE_ABS = 2e-3, 1e-2, 1e-4
+
+
+class Run:
+    def __init__(self, w, device="cuda", max_seqs=64, max_decode_branches=16, max_splits=16,
+                 max_pages=None, pool_seed=None, cache_layers=64):
+        self.w = w
+        self.device = device
+        seed = w.seed if pool_seed is None else pool_seed
+        self.pool = stpkg.Pool(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                               head_dim=w.head_dim, n_blocks=w.n_blocks, seed=seed, max_seqs=max_seqs,
+                               max_pages=max_pages or min(w.n_blocks, 1 << 16),
+                               max_decode_branches=max_decode_branches, max_splits=max_splits,
+                               device=device)
+        self.ref = R.RefPool(w.n_blocks, seed, max_seqs=max_seqs)
+        self.hist = {}
+        self.handle = {}
+        self.sizes = {}
+        self._cache = OrderedDict()
+        self._cache_cap = cache_layers
+
+    # -- operations (library and reference in lock-step) ---------------------
+    def create(self):
+        rid = self.ref.create()
+        self.handle[rid] = self.pool.seq_create()
+        self.hist[rid] = []
+        return rid
+
+    def fork(self, rid, n_aux=4):
+        kids = self.ref.fork(rid, n_aux)
+        for k, h in zip(kids, self.pool.fork(self.handle[rid], n_aux)):
+            self.handle[k] = h
+            self.hist[k] = list(self.hist[rid])
+        return kids
+
+    def append(self, rids, n_tok, tag):
+        w = self.w
+        n = len(rids)
+        k, v = kv_rows(w, tag, n * n_tok, device=self.device)
+        shape = (w.n_layers, n, n_tok, w.n_kv_heads, w.head_dim)
+        self.pool.append_kv([self.handle[r] for r in rids], k.view(shape), v.view(shape))
+        self.ref.append(rids, n_tok)
+        self.sizes[tag] = n * n_tok
+        for i, r in enumerate(rids):
+            self.hist[r].append((tag, i * n_tok, n_tok))
+
+    def decode(self, rids, tag):
+        w = self.w
+        q = queries(w, tag, len(rids), device=self.device)
+        o, lse = self.pool.decode_attn([self.handle[r] for r in rids], q)
+        return q, o, lse
+
+    def merge(self, rid, T, tag):
+        w = self.w
+        k, v = kv_rows(w, tag, T, device=self.device)
+        q = queries(w, ("merge_q",) + tuple(tag), T, device=self.device)
+        L0 = self.ref.seqs[rid].length
+        o, lse = self.pool.merge(self.handle[rid], q, k, v)
+        self.ref.merge(rid, T)
+        self.sizes[tag] = T
+        self.hist[rid].append((tag, 0, T))
+        return q, o, lse, L0
+
+    def release(self, rid):
+        self.ref.release(rid)
+        self.pool.release(self.handle[rid])
+
+    # -- oracle side ----------------------------------------------------------
+    def _rows(self, tag, layer):
+        key = (tag, layer)
+        if key in self._cache:
+            self._cache.move_to_end(key)
+            return self._cache[key]
+        k, v = kv_rows(self.w, tag, self.sizes[tag], device=self.device, layers=[layer])
+        val = (k[0].cpu(), v[0].cpu())
+        self._cache[key] = val
+        if len(self._cache) > self._cache_cap:
+            self._cache.popitem(last=False)
+        return val
+
+    def context(self, rid, layer):
+        """(K, V) bf16 [n, Hkv, D] of sequence rid at `layer`, in logical order."""
+        ks, vs = [], []
+        for tag, off, cnt in self.hist[rid]:
+            k, v = self._rows(tag, layer)
+            ks.append(k[off:off + cnt])
+            vs.append(v[off:off + cnt])
+        return torch.cat(ks), torch.cat(vs)
+
+    def oracle_decode(self, rids, q, layer):
+        """float64 O [n_br, Hq, D], LSE [n_br, Hq] for one layer."""
+        outs = [A.decode(q[layer, i].cpu(), *self.context(r, layer)) for i, r in enumerate(rids)]
+        return np.stack([o for o, _ in outs]), np.stack([l for _, l in outs])
+
+    def check_tables(self):
+        assert self.pool.refcounts() == self.ref.ref
+        assert self.pool.free_list() == list(self.ref.free)
+        for rid in self.ref.live():
+            table, n = self.pool.block_table(self.handle[rid])
+            assert table == self.ref.seqs[rid].table, rid
+            assert n == self.ref.seqs[rid].length
+
+
+def compare(o_gpu, lse_gpu, o_ref, lse_ref, what=""):
+    """Element-wise check against the oracle; returns (max_abs, max_rel, max_lse)."""
+    o = o_gpu.double().cpu().numpy() if isinstance(o_gpu, torch.Tensor) else o_gpu
+    l = lse_gpu.double().cpu().numpy() if isinstance(lse_gpu, torch.Tensor) else lse_gpu
+    assert np.isfinite(o).all() and np.isfinite(l).all(), what
+    err = np.abs(o - o_ref)
+    bad = err > O_ABS + O_REL * np.abs(o_ref)
+    lerr = np.abs(l - lse_ref)
+    rel = err / np.maximum(np.abs(o_ref), 1e-30)
+    assert not bad.any(), f"{what}: {bad.sum()} O elements out of tolerance, max abs {err.max():.3e}"
+    assert (lerr <= LSE_ABS).all(), f"{what}: max lse err {lerr.max():.3e}"
+    return float(err.max()), float(rel[np.abs(o_ref) > 1e-3].max(initial=0.0)), float(lerr.max())

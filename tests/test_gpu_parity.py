@@ -1,0 +1,301 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 oracle on
+the same seeded inputs.  Block tables, refcounts and the free list must match
+bit-exactly; O within 2e-3 + 1e-2|ref| element-wise, LSE within 1e-4."""
+import numpy as np
+import pytest
+import torch
+
+from fg_harness import Run, compare
+from oracle import attention as A
+from workloads import Workload, get
+
+pytestmark = pytest.mark.gpu
+
+CHUNK = 8192  # prefix rows per append call
+
+
+def _prefix(run, rid, P, tag):
+    for c0 in range(0, P, CHUNK):
+        run.append([rid], min(CHUNK, P - c0), (tag, c0))
+
+
+def _run(w, **kw):
+    lim = dict(w.limits)
+    lim.update(kw)
+    return Run(w, **lim)
+
+
+def test_cfg1_tiny_fork_group(stlib):
+    w = get(1)
+    run = _run(w)
+    m = run.create()
+    run.append([m], w.prefix[0], ("prefix",))
+    aux = run.fork(m, w.n_aux)
+    for i, (a, s) in enumerate(zip(aux, w.suffix[0][1:])):
+        run.append([a], s, ("suffix", i))
+    rids = [m] + aux
+    q, o, lse = run.decode(rids, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    o_ref, l_ref = run.oracle_decode(rids, q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "cfg1")
+    # the prefix pages are permuted in physical memory
+    table = run.pool.block_table(run.handle[m])[0]
+    assert table != sorted(table)
+
+
+def test_cfg2_single_agent_turn(stlib):
+    w = get(2)
+    run = _run(w)
+    m = run.create()
+    run.append([m], w.prefix[0], ("prefix",))
+    aux = run.fork(m, w.n_aux)
+    rids = [m] + aux
+    run.append(rids, w.suffix[0][0], ("suffix",))
+    checks = {0, 1, 15, 16, 100, w.steps - 1}
+    for step in range(w.steps):
+        run.append(rids, 1, ("step", step))
+        q, o, lse = run.decode(rids, ("q", step))
+        if step in checks:
+            o_ref, l_ref = run.oracle_decode(rids, q, 0)
+            compare(o[0], lse[0], o_ref, l_ref, f"cfg2 step {step}")
+    run.pool.sync()
+    run.check_tables()
+
+
+def test_cfg3_batched_agent_serving(stlib):
+    w = get(3)
+    run = _run(w)
+    groups = []
+    for t in range(w.n_tasks):
+        m = run.create()
+        _prefix(run, m, w.prefix[t], ("prefix", t))
+        aux = run.fork(m, w.n_aux)
+        br = [m] + aux
+        for b, (rid, s) in enumerate(zip(br, w.suffix[t])):
+            if s:
+                run.append([rid], s, ("suffix", t, b))
+        groups.append(br)
+    rids = [r for g in groups for r in g]
+    run.append(rids, 1, ("step",))
+    q, o, lse = run.decode(rids, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    o_ref, l_ref = run.oracle_decode(rids, q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "cfg3")
+
+
+def test_cfg4_long_trajectory_sampled_layers(stlib):
+    w = get(4)
+    run = _run(w, cache_layers=48)
+    groups = []
+    for t in range(w.n_tasks):
+        m = run.create()
+        _prefix(run, m, w.prefix[t], ("prefix", t))
+        aux = run.fork(m, w.n_aux)
+        br = [m] + aux
+        for b, (rid, s) in enumerate(zip(br, w.suffix[t])):
+            if s:
+                run.append([rid], s, ("suffix", t, b))
+        groups.append(br)
+    rids = [r for g in groups for r in g]
+    run.append(rids, 1, ("step",))
+    q, o, lse = run.decode(rids, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    for layer in (0, w.n_layers - 1):
+        o_ref, l_ref = run.oracle_decode(rids, q, layer)
+        compare(o[layer], lse[layer], o_ref, l_ref, f"cfg4 layer {layer}")
+
+
+def test_cfg5_full_cycle_sampled(stlib):
+    w = get(5)
+    run = _run(w, cache_layers=32)
+    mains = []
+    for t in range(w.n_tasks):
+        m = run.create()
+        _prefix(run, m, w.prefix[t], ("prefix", t))
+        mains.append(m)
+    rng = np.random.default_rng(5)
+    check_steps = {0, 255, w.steps - 1}
+    for turn in range(w.turns):
+        singles = [run.create() for _ in range(w.singletons)]
+        for i in range(0, w.singletons, 8):
+            run.append(singles[i:i + 8], w.singleton_len, ("single", turn, i))
+        groups = [[m] + run.fork(m, w.n_aux) for m in mains]
+        rids = [r for g in groups for r in g] + singles
+        for step in range(w.steps):
+            run.append(rids, 1, ("step", turn, step))
+            q, o, lse = run.decode(rids, ("q", turn, step))
+            if step in check_steps:
+                layer = (7 * turn + step) % w.n_layers
+                sample = groups[turn % w.n_tasks] + singles[:2]
+                idx = [rids.index(r) for r in sample]
+                o_ref, l_ref = run.oracle_decode(sample, q[:, idx], layer)
+                compare(o[layer][idx], lse[layer][idx], o_ref, l_ref, f"cfg5 turn {turn} step {step}")
+        for t, m in enumerate(mains):
+            qm, om, lm, L0 = run.merge(m, w.merge_tokens, ("merge", turn, t))
+            if t == turn % w.n_tasks:
+                layer = (3 * turn + 1) % w.n_layers
+                rows = sorted({0, 1, 63, 64, w.merge_tokens - 1, *rng.integers(0, w.merge_tokens, 6).tolist()})
+                k, v = run.context(m, layer)
+                o_ref, l_ref = A.merge_prefill(qm[layer].cpu(), k, v, L0, rows=rows)
+                compare(om[layer][rows], lm[layer][rows], o_ref, l_ref, f"cfg5 merge turn {turn}")
+        for g in groups:
+            for a in g[1:]:
+                run.release(a)
+        for s in singles:
+            run.release(s)
+        run.pool.sync()
+        run.check_tables()
+
+
+# ---- edge cases on small shapes -------------------------------------------
+
+def _small(D, Hq, Hkv, n_blocks=512, L=2, seed=11, scale=1.0):
+    return Workload(name=f"edge_{D}_{Hq}_{Hkv}", n_layers=L, n_q_heads=Hq, n_kv_heads=Hkv,
+                    head_dim=D, n_blocks=n_blocks, seed=seed, value_scale=scale)
+
+
+@pytest.mark.parametrize("D,Hq,Hkv,n_aux,P,suffix", [
+    (64, 8, 2, 4, 512, (0, 16, 33, 47, 64)),
+    (128, 32, 8, 1, 1000, (5, 0)),
+    (128, 8, 8, 7, 777, (1, 2, 3, 0, 16, 17, 31, 100)),      # G = 1, eight branches
+    (128, 64, 8, 4, 300, (0, 1, 15, 16, 17)),                # G = 8, 40 stacked rows
+    (128, 64, 8, 8, 4100, (3,) * 9),                         # 9 x 8 rows -> two subgroups
+    (128, 16, 1, 3, 2000, (0, 9, 0, 40)),                    # G = 16, 64 rows
+    (128, 32, 1, 1, 100, (0, 0)),                            # G = 32, no suffixes
+    (64, 4, 1, 0, 50, (0,)),                                 # a lone main thread
+    (64, 12, 3, 2, 16, (0, 1, 2)),                           # one-page prefix
+    (128, 32, 8, 4, 15, (0, 1, 2, 3, 4)),                    # prefix shorter than a page
+])
+def test_shapes(stlib, D, Hq, Hkv, n_aux, P, suffix):
+    w = _small(D, Hq, Hkv)
+    run = Run(w, max_seqs=16, max_decode_branches=16, max_splits=8)
+    m = run.create()
+    run.append([m], P, ("prefix",))
+    br = [m] + (run.fork(m, n_aux) if n_aux else [])
+    for b, (rid, s) in enumerate(zip(br, suffix)):
+        if s:
+            run.append([rid], s, ("suffix", b))
+    q, o, lse = run.decode(br, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    for layer in range(w.n_layers):
+        o_ref, l_ref = run.oracle_decode(br, q, layer)
+        compare(o[layer], lse[layer], o_ref, l_ref, f"layer {layer}")
+
+
+def test_many_splits_on_a_long_singleton(stlib):
+    w = _small(128, 32, 8, n_blocks=4096, L=1)
+    run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=32)
+    a = run.create()
+    for c0 in range(0, 40000, 8000):
+        run.append([a], 8000, ("ctx", c0))
+    b = run.create()
+    run.append([b], 3, ("short",))
+    q, o, lse = run.decode([a, b], ("q",))
+    o_ref, l_ref = run.oracle_decode([a, b], q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "long singleton")
+
+
+def test_stale_nan_pool_memory_does_not_leak(stlib):
+    w = _small(128, 32, 8, n_blocks=256, L=1)
+    run = Run(w, max_seqs=8, max_decode_branches=8, max_splits=8)
+    run.pool.k_pool.fill_(float("nan"))
+    run.pool.v_pool.fill_(float("nan"))
+    m = run.create()
+    run.append([m], 999, ("prefix",))
+    br = [m] + run.fork(m, 4)
+    for b, rid in enumerate(br):
+        run.append([rid], b * 5 + 1, ("suffix", b))
+    q, o, lse = run.decode(br, ("q",))
+    o_ref, l_ref = run.oracle_decode(br, q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "nan pool")
+    T = 37
+    qm, om, lm, L0 = run.merge(m, T, ("merge",))
+    k, v = run.context(m, 0)
+    o_ref, l_ref = A.merge_prefill(qm[0].cpu(), k, v, L0)
+    compare(om[0], lm[0], o_ref, l_ref, "nan pool merge")
+
+
+def test_outputs_do_not_depend_on_page_placement(stlib):
+    outs = []
+    for seed in (1, 2):
+        w = _small(128, 32, 8, n_blocks=512, L=1)
+        run = Run(w, max_seqs=8, max_decode_branches=8, max_splits=8, pool_seed=seed)
+        m = run.create()
+        run.append([m], 3000, ("prefix",))
+        br = [m] + run.fork(m, 4)
+        for b, rid in enumerate(br[1:], start=1):
+            run.append([rid], 7 * b, ("suffix", b))
+        q, o, lse = run.decode(br, ("q",))
+        outs.append((o.clone(), lse.clone(), run.pool.block_table(run.handle[m])[0]))
+    assert outs[0][2] != outs[1][2]
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+def test_copy_on_write_keeps_siblings_intact(stlib):
+    w = _small(64, 8, 2, n_blocks=128, L=2)
+    run = Run(w, max_seqs=8, max_decode_branches=8, max_splits=8)
+    m = run.create()
+    run.append([m], 40, ("prefix",))      # two full pages + 8 rows in a shared page
+    aux = run.fork(m, 2)
+    run.append([aux[0]], 20, ("a0",))     # copies the shared page, then writes
+    run.append([m], 3, ("m",))            # copies too (still shared with aux[1])
+    run.append([aux[1]], 1, ("a1",))      # last holder: writes in place
+    br = [m] + aux
+    q, o, lse = run.decode(br, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    for layer in range(2):
+        o_ref, l_ref = run.oracle_decode(br, q, layer)
+        compare(o[layer], lse[layer], o_ref, l_ref, f"cow layer {layer}")
+
+
+@pytest.mark.parametrize("D,Hq,Hkv,L0,T", [
+    (128, 32, 8, 1000, 1), (128, 32, 8, 1000, 5), (128, 32, 8, 1003, 17), (128, 64, 8, 512, 100),
+    (64, 8, 2, 77, 64), (128, 8, 8, 33, 130), (128, 32, 1, 16, 9),
+])
+def test_merge_prefill(stlib, D, Hq, Hkv, L0, T):
+    w = _small(D, Hq, Hkv, n_blocks=512, L=2)
+    run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=8)
+    m = run.create()
+    run.append([m], L0, ("ctx",))
+    aux = run.fork(m, 1)                  # a live sibling shares main's pages
+    qm, om, lm, L0r = run.merge(m, T, ("merge",))
+    assert L0r == L0
+    run.pool.sync()
+    run.check_tables()
+    for layer in range(2):
+        k, v = run.context(m, layer)
+        o_ref, l_ref = A.merge_prefill(qm[layer].cpu(), k, v, L0)
+        compare(om[layer], lm[layer], o_ref, l_ref, f"merge layer {layer}")
+    # the sibling still sees only the pre-merge context
+    q, o, lse = run.decode(aux, ("q",))
+    o_ref, l_ref = run.oracle_decode(aux, q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "sibling after merge")
+
+
+def test_merge_of_one_row_equals_decode_after_append(stlib):
+    w = _small(128, 32, 8, n_blocks=256, L=1)
+    run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=8)
+    m = run.create()
+    run.append([m], 500, ("ctx",))
+    qm, om, lm, _ = run.merge(m, 1, ("merge",))
+    o, lse = run.pool.decode_attn([run.handle[m]], qm.view(1, 1, w.n_q_heads, w.head_dim).contiguous())
+    torch.testing.assert_close(o[0, 0], om[0, 0], atol=2e-3, rtol=1e-2)
+    torch.testing.assert_close(lse[0, 0], lm[0, 0], atol=1e-4, rtol=0)
+
+
+def test_merge_of_nothing_changes_nothing(stlib):
+    w = _small(128, 32, 8, n_blocks=64, L=1)
+    run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=8)
+    m = run.create()
+    run.append([m], 20, ("ctx",))
+    snap = (run.pool.refcounts(), run.pool.free_list(), run.pool.block_table(run.handle[m]))
+    e = torch.empty((1, 0, w.n_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    kv = torch.empty((1, 0, w.n_kv_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    run.pool.merge(run.handle[m], e, kv, kv)
+    assert snap == (run.pool.refcounts(), run.pool.free_list(), run.pool.block_table(run.handle[m]))
+    run.pool.sync()

@@ -31,7 +31,8 @@ class Workload:
     merge_tokens: int = 0     # rows appended to main by st_merge each turn
     singletons: int = 0       # unforked decode-only sequences
     singleton_len: int = 0
-    extra: dict = field(default_factory=dict)
+    # pool capacities used by both the tests and the bench (launch configuration)
+    limits: dict = field(default_factory=dict)
 
     @property
     def group(self):
@@ -47,14 +48,16 @@ def _tiny():
     return Workload(
         name="tiny_fork_group", n_layers=1, n_q_heads=8, n_kv_heads=2, head_dim=64,
         n_blocks=64, seed=0, value_scale=0.125, n_tasks=1,
-        prefix=(512,), suffix=((0, 16, 33, 47, 64),), steps=0)
+        prefix=(512,), suffix=((0, 16, 33, 47, 64),), steps=0,
+        limits=dict(max_seqs=8, max_decode_branches=5, max_splits=8, max_pages=64))
 
 
 def _single_turn():
     return Workload(
         name="single_agent_turn", n_layers=1, n_q_heads=32, n_kv_heads=8, head_dim=128,
         n_blocks=1024, seed=1, n_tasks=1, prefix=(8192,),
-        suffix=((256, 256, 256, 256, 256),), steps=256)
+        suffix=((256, 256, 256, 256, 256),), steps=256,
+        limits=dict(max_seqs=8, max_decode_branches=5, max_splits=16, max_pages=1024))
 
 
 def _batched():
@@ -65,17 +68,20 @@ def _batched():
     # 2 GiB of K+V for one layer: 32768 blocks of 16 tokens x 8 heads x 128 x bf16 x {K,V}
     return Workload(
         name="batched_agent_serving", n_layers=1, n_q_heads=32, n_kv_heads=8, head_dim=128,
-        n_blocks=32768, seed=2, n_tasks=16, prefix=P, suffix=S, steps=1)
+        n_blocks=32768, seed=2, n_tasks=16, prefix=P, suffix=S, steps=1,
+        limits=dict(max_seqs=96, max_decode_branches=80, max_splits=16, max_pages=2304))
 
 
 def _long():
     import numpy as np
     rng = np.random.default_rng(3)
     S = tuple(tuple(int(x) for x in rng.integers(0, 2048, size=5, endpoint=True)) for _ in range(4))
-    pages = sum(131072 // 16 + sum((s + 16 + 15) // 16 + 1 for s in row) for row in S)
+    # room for every suffix plus 256 decode steps per branch
+    pages = sum(131072 // 16 + sum((s + 256 + 15) // 16 + 1 for s in row) for row in S)
     return Workload(
         name="long_trajectory_agent", n_layers=32, n_q_heads=64, n_kv_heads=8, head_dim=128,
-        n_blocks=pages + 256, seed=3, n_tasks=4, prefix=(131072,) * 4, suffix=S, steps=1)
+        n_blocks=pages + 64, seed=3, n_tasks=4, prefix=(131072,) * 4, suffix=S, steps=1,
+        limits=dict(max_seqs=24, max_decode_branches=20, max_splits=32, max_pages=8192 + 160))
 
 
 def _cycle():
@@ -86,7 +92,8 @@ def _cycle():
         name="full_fork_decode_merge_cycle", n_layers=32, n_q_heads=32, n_kv_heads=8,
         head_dim=128, n_blocks=8 * per_task + singles + 256, seed=4, n_tasks=8,
         prefix=(16384,) * 8, suffix=((0, 0, 0, 0, 0),) * 8, steps=512, turns=5,
-        merge_tokens=2048, singletons=64, singleton_len=2048)
+        merge_tokens=2048, singletons=64, singleton_len=2048,
+        limits=dict(max_seqs=112, max_decode_branches=104, max_splits=16, max_pages=2048))
 
 
 CONFIGS = {
