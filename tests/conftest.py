@@ -31,3 +31,19 @@ def stlib():
     import paper_2608_13667_gb300 as stpkg
     stpkg.build()
     return stpkg
+
+
+@pytest.fixture(autouse=True)
+def _release_device_memory(request):
+    """Return pooled device memory between GPU tests (the full-size workloads
+    each hold tens of GB)."""
+    yield
+    if request.node.get_closest_marker("gpu"):
+        import gc
+        gc.collect()
+        try:
+            import torch
+            if torch.cuda.is_available():
+                torch.cuda.empty_cache()
+        except ImportError:
+            pass
