@@ -181,6 +181,48 @@ typedef struct {
 ST_API st_status st_profile_enable(st_pool* pool, int enable);
 ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, int* n);
 
+/* ---- Allocation-free decode ------------------------------------------------
+ * The paper has no counterpart to this call; it exists for callers that
+ * cannot allocate device memory: code running inside a host framework that
+ * owns every device allocation and forbids new ones after start-up,
+ * real-time serving loops that must not allocate on the hot path, and plugins
+ * that are handed input and output pointers but no allocator.  Such callers
+ * cannot supply the workspace st_pool_create needs, so this call takes only
+ * inputs and outputs and allocates nothing (no cudaMalloc, no cudaFree, no
+ * allocating library routine).  It runs the same kernels as st_decode_attn.
+ *
+ * Its scratch -- the per-call plan, a device copy of the page tables and the
+ * split-KV partials -- lives in a static device array of
+ * ST_NOALLOC_SCRATCH_BYTES (16 MiB) that every GPU loading the library holds
+ * until the process exits.  The first call on a device looks up that array's
+ * device address (once per device, with the device current); make that
+ * first call before any stream capture.  Every call reuses the array, so
+ * calls that overlap on the GPU (different streams without ordering) race.
+ *
+ * geom:        pool geometry (n_layers, n_q_heads, n_kv_heads, head_dim,
+ *              page_size = 16, n_blocks); other fields are ignored.
+ * k_pool/v_pool: device bf16 [n_layers][n_blocks][n_kv_heads][16][head_dim]
+ *              (the st_pool_create layout), 16-byte aligned.
+ * page_table:  HOST int32 [n_br][table_stride], each branch's physical page
+ *              ids in logical order; ids must lie in [0, n_blocks).
+ * seq_len:     HOST int32 [n_br], tokens in each branch's context (>= 1,
+ *              ceil(len / 16) <= table_stride).
+ * q, o, lse:   as st_decode_attn, on the current device.
+ * Branches whose tables start on the same physical page are treated as one
+ * fork group: their common full pages are read once for the group.
+ * Returns ST_ERR_INVALID for bad arguments or n_br > ST_NOALLOC_MAX_BRANCHES,
+ * and ST_ERR_OOM when the call needs more than the static scratch:
+ *   256-byte-rounded 37 KiB plan + 4*n_br*table_stride
+ *   + 4*n_layers*n_br*n_q_heads*16*(head_dim + 1) bytes > 16 MiB.
+ * The work runs on `stream`; device-side bounds checks skip a bad page id
+ * (it reads as zeros) without reporting it. */
+#define ST_NOALLOC_SCRATCH_BYTES (16u << 20)
+#define ST_NOALLOC_MAX_BRANCHES 64
+ST_API st_status st_decode_attn_noalloc(const st_config* geom, const void* k_pool, const void* v_pool,
+                                        const int32_t* page_table, int table_stride,
+                                        const int32_t* seq_len, int n_br, const void* q, float* o,
+                                        float* lse, void* stream);
+
 ST_API const char* st_status_str(st_status s);
 ST_API const char* st_last_error(st_pool* pool);
 

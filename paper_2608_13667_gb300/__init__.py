@@ -83,6 +83,7 @@ def lib():
         "st_sync": (I, [P, VP]),
         "st_profile_enable": (I, [P, I]),
         "st_profile_read": (I, [P, ctypes.POINTER(StKernelStat), I, ctypes.POINTER(I)]),
+        "st_decode_attn_noalloc": (I, [ctypes.POINTER(StConfig), VP, VP, i32p, I, i32p, I, VP, VP, VP, VP]),
         "st_status_str": (ctypes.c_char_p, [I]),
         "st_last_error": (ctypes.c_char_p, [P]),
     }
@@ -313,3 +314,24 @@ def st_release(pool, seq):
 
 def st_sync(pool, stream=None):
     return pool.sync(stream)
+
+
+def st_decode_attn_noalloc(geom, k_pool, v_pool, page_tables, seq_len, q, o, lse, stream=None):
+    """Allocation-free decode (see include/st.h): geom is a StConfig, k_pool/v_pool
+    the bf16 KV tensors, page_tables a list of per-branch page-id lists (host),
+    seq_len per-branch token counts, q/o/lse device tensors as for
+    st_decode_attn.  Returns the status code."""
+    import torch
+    n_br = len(seq_len)
+    stride = max(1, max(len(t) for t in page_tables))
+    table = (ctypes.c_int32 * (n_br * stride))()
+    for i, t in enumerate(page_tables):
+        for j, b in enumerate(t):
+            table[i * stride + j] = b
+    lens = (ctypes.c_int32 * n_br)(*[int(x) for x in seq_len])
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    return lib().st_decode_attn_noalloc(ctypes.byref(geom), ctypes.c_void_p(k_pool.data_ptr()),
+                                        ctypes.c_void_p(v_pool.data_ptr()), table, stride, lens, n_br,
+                                        ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(o.data_ptr()),
+                                        ctypes.c_void_p(lse.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
