@@ -66,7 +66,7 @@ typedef struct st_pool st_pool;
 typedef struct {
   int32_t n_layers;
   int32_t n_q_heads;
-  int32_t n_kv_heads;          /* must divide n_q_heads; G = n_q_heads / n_kv_heads <= 64 */
+  int32_t n_kv_heads;          /* must divide n_q_heads; G = n_q_heads / n_kv_heads <= 48 */
   int32_t head_dim;            /* 64 or 128 */
   int32_t page_size;           /* tokens per page; must be 16 */
   int32_t max_seqs;            /* live sequences at once (handle slots) */

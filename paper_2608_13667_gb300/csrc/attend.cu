@@ -8,10 +8,10 @@
 // query heads of the KV head -- so each prefix page crosses HBM once per
 // group instead of once per branch.
 //
-// CTA layout (160 threads): warps 0..3 compute, warp 4 loads.
+// CTA layout (128 threads): warps 0..2 compute, warp 3 loads; 3 CTAs per SM.
 //   * Loader: reads page ids from the block table (32 at a time, one batch
 //     ahead) and issues one 2 KiB TMA tensor copy per (page, 64-wide half of
-//     the head, K|V) into a 3-stage ring of 4-page stages, signalling a
+//     the head, K|V) into a 2-stage ring of 4-page stages, signalling a
 //     per-stage mbarrier with the byte count.
 //   * Compute warp w owns query rows [16w, 16w+16).  Per stage it forms
 //     S = Q K^T on the tensor cores (mma.sync m16n8k16 bf16 -> fp32; K
@@ -36,8 +36,8 @@ namespace st {
 namespace {
 
 constexpr int kPPS = 4;            // pages per pipeline stage (64 keys)
-constexpr int kStages = 3;
-constexpr int kComputeWarps = 4;   // up to 64 stacked query rows
+constexpr int kStages = 2;
+constexpr int kComputeWarps = 3;   // up to 48 stacked query rows
 constexpr int kThreads = (kComputeWarps + 1) * 32;
 constexpr float kLn2 = 0.69314718055994530942f;
 
@@ -64,7 +64,7 @@ __device__ __forceinline__ uint32_t ld_u32(const __nv_bfloat16* p) {
 }
 
 template <int D, bool kCausal>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 3)
     attend_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                   const AttnParams p) {
   using Geo = Geometry<D>;

@@ -33,7 +33,7 @@ constexpr size_t kScratchBytes = ST_NOALLOC_SCRATCH_BYTES;
 constexpr int kMaxBranches = ST_NOALLOC_MAX_BRANCHES;
 constexpr int kMaxItems = 1024;
 constexpr int kSplitStride = 16;  // partial slots per (layer, branch, head)
-constexpr int kMaxRows = 64;      // stacked query rows per CTA
+constexpr int kMaxRows = 48;      // stacked query rows per CTA
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];

@@ -28,7 +28,7 @@ namespace {
 
 constexpr int kStageSlots = 8;
 constexpr size_t kStageSlotBytes = 2u << 20;  // 2 MiB per plan
-constexpr int kMaxAttnRows = 64;              // stacked query rows per CTA
+constexpr int kMaxAttnRows = 48;              // stacked query rows per CTA
 
 enum KernelId { kKTable = 0, kKAppend, kKDecode, kKCombine, kKMerge, kNumKernels };
 const char* const kKernelNames[kNumKernels] = {"table_update", "append_kv", "decode_partial",
@@ -49,7 +49,7 @@ bool config_valid(const st_config* c, std::string* why) {
   if (c->n_layers < 1) return bad("n_layers must be >= 1");
   if (c->n_kv_heads < 1 || c->n_q_heads < 1 || c->n_q_heads % c->n_kv_heads != 0)
     return bad("n_kv_heads must divide n_q_heads");
-  if (c->n_q_heads / c->n_kv_heads > kMaxAttnRows) return bad("n_q_heads / n_kv_heads must be <= 64");
+  if (c->n_q_heads / c->n_kv_heads > kMaxAttnRows) return bad("n_q_heads / n_kv_heads must be <= 48");
   if (c->head_dim != 64 && c->head_dim != 128) return bad("head_dim must be 64 or 128");
   if (c->page_size != kPageTokens) return bad("page_size must be 16");
   if (c->max_seqs < 1) return bad("max_seqs must be >= 1");
