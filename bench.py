@@ -38,7 +38,9 @@ def _peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def _dist():
+def _dist(backend=None):
+    """(rank, world, local rank).  One process per GPU under torchrun; NCCL on
+    GPUs, gloo when asked (the CPU tests of the multi-rank path)."""
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     if ws <= 1:
         return 0, 1, 0
@@ -46,17 +48,23 @@ def _dist():
     import torch.distributed as dist
     rank = int(os.environ["RANK"])
     local = int(os.environ.get("LOCAL_RANK", rank))
-    torch.cuda.set_device(local)
-    dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    backend = backend or ("nccl" if torch.cuda.is_available() else "gloo")
+    if backend == "nccl":
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        dist.init_process_group("gloo")
     return rank, ws, local
 
 
-def _barrier_max(x, ws):
+def _allreduce_max(x, ws):
+    """Max of a float over ranks (timings: the slowest rank sets the time)."""
     if ws <= 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
 
@@ -217,7 +225,7 @@ def run_ours(args, rank, ws, local):
     pool.sync()
     stats = pool.profile_read()
     pool.profile_enable(False)
-    ms_max = _barrier_max(ms, ws)
+    ms_max = _allreduce_max(ms, ws)
 
     # end-to-end through the public API with host buffers: H2D of the step's
     # q and new K/V rows from pinned memory, D2H of O and LSE, every step
@@ -240,7 +248,7 @@ def run_ours(args, rank, ws, local):
         ho.copy_(o, non_blocking=True)
         hl.copy_(lse, non_blocking=True)
     torch.cuda.synchronize(dev)
-    e2e_s = _barrier_max(time.perf_counter() - t0, ws)
+    e2e_s = _allreduce_max(time.perf_counter() - t0, ws)
     h2d = hq[0].numel() * 2 + hk[0].numel() * 2 * 2
     d2h = ho.numel() * 4 + hl.numel() * 4
 

@@ -16,7 +16,7 @@ from oracle import attention as A
 from oracle import pool as R
 from workloads import kv_rows, queries
 
-# Tolerances (benchmark spec): elementwise |gpu - oracle| <= 2e-3 + 1e-2 |oracle|
+# Tolerances of the parity target: element-wise |gpu - oracle| <= 2e-3 + 1e-2 |oracle|
 # for O; |gpu - oracle| <= 1e-4 for the log-sum-exp.
 O_ABS, O_REL, LSE_ABS = 2e-3, 1e-2, 1e-4
 
