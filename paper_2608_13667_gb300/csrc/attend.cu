@@ -1,4 +1,4 @@
-// Paged attention over block tables: decode partials and the merge prefill.
+// Paged decode attention over block tables (split-KV partials + combine).
 //
 // Section 3.3 of the paper: all branches share the prompt prefix up to R_t, so
 // the prefix KV is reused across every decoding stream; Section 4.4: branch
@@ -19,9 +19,8 @@
 //     softmax in the log2 domain (row max/sum via quad shuffles; the
 //     accumulator is rescaled only when some row max grows), rounds P to bf16
 //     and accumulates O += P V (V fragments by ldmatrix.trans).
-// Decode writes a normalised partial (O_i, lse_i) per row into its split
-// slot for the log-sum-exp combine; the merge (causal, Section 3.5: thought
-// row i sees main's rows [0, L0 + i]) writes final O and lse.
+// Each CTA writes a normalised partial (O_i, lse_i) per row into its split
+// slot; combine_kernel merges a branch's partials by log-sum-exp.
 //
 // Key rows past the valid length of a partially filled last page may hold
 // stale data; their scores are masked to -inf and their V values are zeroed
@@ -63,7 +62,7 @@ __device__ __forceinline__ uint32_t ld_u32(const __nv_bfloat16* p) {
   return *reinterpret_cast<const uint32_t*>(p);
 }
 
-template <int D, bool kCausal>
+template <int D>
 __global__ void __launch_bounds__(kThreads, 3)
     attend_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                   const AttnParams p) {
@@ -80,27 +79,12 @@ __global__ void __launch_bounds__(kThreads, 3)
   const int layer = blockIdx.z;
 
   // ---- what this CTA reads and for whom -----------------------------------
-  int slot, page_begin, n_pages, n_valid_keys, n_rows, min_limit, row_base = 0;
-  AttnItem item{};
-  if (!kCausal) {
-    item = p.items[blockIdx.x];
-    slot = item.slot;
-    page_begin = item.page_begin;
-    n_pages = item.n_pages;
-    n_valid_keys = item.n_tokens;
-    n_rows = item.n_members * p.G;
-    min_limit = item.n_tokens;
-  } else {
-    slot = p.slot;
-    page_begin = 0;
-    row_base = blockIdx.x * (kComputeWarps * 16);
-    n_rows = min(kComputeWarps * 16, p.T * p.G - row_base);
-    const int t_first = row_base / p.G;
-    const int t_last = (row_base + n_rows - 1) / p.G;
-    n_pages = (p.L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
-    n_valid_keys = p.L0 + p.T;
-    min_limit = p.L0 + t_first + 1;
-  }
+  const AttnItem item = p.items[blockIdx.x];
+  const int slot = item.slot;
+  const int page_begin = item.page_begin;
+  const int n_pages = item.n_pages;
+  const int n_valid_keys = item.n_tokens;  // keys past this in the last page are stale
+  const int n_rows = item.n_members * p.G;
   const int n_cw = (n_rows + 15) >> 4;
   const int n_stages = (n_pages + kPPS - 1) / kPPS;
 
@@ -119,9 +103,8 @@ __global__ void __launch_bounds__(kThreads, 3)
       prefetch_tensormap(&kmap);
       prefetch_tensormap(&vmap);
     }
-    // Decode streams each page once: keep it out of L2's way.  The merge's
-    // CTAs of one (layer, head) all walk the same pages: default policy.
-    const uint64_t policy = kCausal ? l2_policy_evict_last() : l2_policy_evict_first();
+    // each page is streamed once: keep it out of L2's way
+    const uint64_t policy = l2_policy_evict_first();
     const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
     int base = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
@@ -184,23 +167,12 @@ __global__ void __launch_bounds__(kThreads, 3)
   const int r1 = r0 + 8;
   const int quad = lane & 3;
 
-  // query row -> (row of q, head) and its key limit
-  auto row_of = [&](int r, int& qrow, int& head) {
-    if (!kCausal) {
-      qrow = p.members[item.member_base + r / p.G];
-      head = kvh * p.G + r % p.G;
-    } else {
-      const int gr = row_base + r;
-      qrow = gr / p.G;
-      head = kvh * p.G + gr % p.G;
-    }
-  };
-  int qrow0 = 0, head0 = 0, qrow1 = 0, head1 = 0;
+  // query row -> (branch of the call, head)
   const bool v0 = r0 < n_rows, v1 = r1 < n_rows;
-  if (v0) row_of(r0, qrow0, head0);
-  if (v1) row_of(r1, qrow1, head1);
-  const int lim0 = kCausal ? (v0 ? p.L0 + qrow0 + 1 : n_valid_keys) : n_valid_keys;
-  const int lim1 = kCausal ? (v1 ? p.L0 + qrow1 + 1 : n_valid_keys) : n_valid_keys;
+  const int qrow0 = v0 ? p.members[item.member_base + r0 / p.G] : 0;
+  const int head0 = v0 ? kvh * p.G + r0 % p.G : 0;
+  const int qrow1 = v1 ? p.members[item.member_base + r1 / p.G] : 0;
+  const int head1 = v1 ? kvh * p.G + r1 % p.G : 0;
 
   uint32_t qa[D / 16][4];
   {
@@ -261,8 +233,8 @@ __global__ void __launch_bounds__(kThreads, 3)
       }
     }
 
-    // scale to the log2 domain, mask, row maxima
-    const bool edge = key0 + kPPS * kPageTokens > min_limit;
+    // scale to the log2 domain, mask keys past the run, row maxima
+    const bool edge = key0 + kPPS * kPageTokens > n_valid_keys;
     float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
     for (int q = 0; q < kPPS; ++q) {
@@ -271,9 +243,8 @@ __global__ void __launch_bounds__(kThreads, 3)
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const int key = key0 + q * kPageTokens + j * 8 + 2 * quad + (e & 1);
-          const int lim = (e < 2) ? lim0 : lim1;
           float x = sc[q][j][e] * sl2;
-          if (q >= np || (edge && key >= lim)) x = -INFINITY;
+          if (q >= np || (edge && key >= n_valid_keys)) x = -INFINITY;
           sc[q][j][e] = x;
         }
         mx0 = fmaxf(mx0, fmaxf(sc[q][j][0], sc[q][j][1]));
@@ -354,28 +325,15 @@ __global__ void __launch_bounds__(kThreads, 3)
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
   const float inv0 = 1.f / l0, inv1 = 1.f / l1;
   float *o0 = nullptr, *o1 = nullptr, *s0 = nullptr, *s1 = nullptr;
-  if (!kCausal) {
-    if (v0) {
-      const int64_t i0 = (((int64_t)layer * p.n_rows_q + qrow0) * p.Hq + head0) * p.max_splits + item.split;
-      o0 = p.out_o + i0 * D;
-      s0 = p.out_lse + i0;
-    }
-    if (v1) {
-      const int64_t i1 = (((int64_t)layer * p.n_rows_q + qrow1) * p.Hq + head1) * p.max_splits + item.split;
-      o1 = p.out_o + i1 * D;
-      s1 = p.out_lse + i1;
-    }
-  } else {
-    if (v0) {
-      const int64_t i0 = ((int64_t)layer * p.T + qrow0) * p.Hq + head0;
-      o0 = p.out_o + i0 * D;
-      s0 = p.out_lse + i0;
-    }
-    if (v1) {
-      const int64_t i1 = ((int64_t)layer * p.T + qrow1) * p.Hq + head1;
-      o1 = p.out_o + i1 * D;
-      s1 = p.out_lse + i1;
-    }
+  if (v0) {
+    const int64_t i0 = (((int64_t)layer * p.n_rows_q + qrow0) * p.Hq + head0) * p.max_splits + item.split;
+    o0 = p.out_o + i0 * D;
+    s0 = p.out_lse + i0;
+  }
+  if (v1) {
+    const int64_t i1 = (((int64_t)layer * p.n_rows_q + qrow1) * p.Hq + head1) * p.max_splits + item.split;
+    o1 = p.out_o + i1 * D;
+    s1 = p.out_lse + i1;
   }
 #pragma unroll
   for (int n = 0; n < D / 8; ++n) {
@@ -436,28 +394,28 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p) {
   if (lane == 0) p.lse[idx] = lse;
 }
 
-template <int D, bool C>
+template <int D>
 cudaError_t launch_attend_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
                             int n_ctas, cudaStream_t s) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attend_kernel<D, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(attend_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Geometry<D>::kSmemBytes);
     if (e != cudaSuccess) return e;
     configured = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  attend_kernel<D, C><<<grid, kThreads, Geometry<D>::kSmemBytes, s>>>(km, vm, p);
+  attend_kernel<D><<<grid, kThreads, Geometry<D>::kSmemBytes, s>>>(km, vm, p);
   return cudaGetLastError();
 }
 
-template <int D, bool C>
+template <int D>
 int ctas_per_sm_t() {
-  cudaError_t e = cudaFuncSetAttribute(attend_kernel<D, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(attend_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Geometry<D>::kSmemBytes);
   if (e != cudaSuccess) return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<D, C>, kThreads,
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<D>, kThreads,
                                                     Geometry<D>::kSmemBytes) != cudaSuccess)
     return 0;
   return n;
@@ -466,18 +424,16 @@ int ctas_per_sm_t() {
 }  // namespace
 
 cudaError_t launch_attend(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
-                          int n_ctas, bool causal, int D, cudaStream_t s) {
+                          int n_ctas, int D, cudaStream_t s) {
   if (n_ctas <= 0) return cudaSuccess;
-  if (D == 128) return causal ? launch_attend_t<128, true>(km, vm, p, n_ctas, s)
-                              : launch_attend_t<128, false>(km, vm, p, n_ctas, s);
-  if (D == 64) return causal ? launch_attend_t<64, true>(km, vm, p, n_ctas, s)
-                             : launch_attend_t<64, false>(km, vm, p, n_ctas, s);
+  if (D == 128) return launch_attend_t<128>(km, vm, p, n_ctas, s);
+  if (D == 64) return launch_attend_t<64>(km, vm, p, n_ctas, s);
   return cudaErrorInvalidValue;
 }
 
-int attend_ctas_per_sm(int D, bool causal) {
-  if (D == 128) return causal ? ctas_per_sm_t<128, true>() : ctas_per_sm_t<128, false>();
-  if (D == 64) return causal ? ctas_per_sm_t<64, true>() : ctas_per_sm_t<64, false>();
+int attend_ctas_per_sm(int D) {
+  if (D == 128) return ctas_per_sm_t<128>();
+  if (D == 64) return ctas_per_sm_t<64>();
   return 0;
 }
 

@@ -452,7 +452,7 @@ ST_API st_status st_pool_create(const st_config* cfg, void* k_pool, void* v_pool
   if (cudaMemset(P->ws, 0, P->lay.staging) != cudaSuccess) return bail(ST_ERR_CUDA);
   if (cudaDeviceGetAttribute(&P->sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
     return bail(ST_ERR_CUDA);
-  P->decode_ctas_per_sm = attend_ctas_per_sm(cfg->head_dim, false);
+  P->decode_ctas_per_sm = attend_ctas_per_sm(cfg->head_dim);
   if (P->decode_ctas_per_sm < 1) return bail(ST_ERR_CUDA);
   if (cudaHostAlloc(reinterpret_cast<void**>(&P->h_stage), (size_t)kStageSlots * kStageSlotBytes,
                     cudaHostAllocDefault) != cudaSuccess)
@@ -718,7 +718,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.max_splits = c.max_splits;
   const int n_items = (int)items.size();
   st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
-    return launch_attend(P->kmap, P->vmap, ap, n_items, false, c.head_dim, s);
+    return launch_attend(P->kmap, P->vmap, ap, n_items, c.head_dim, s);
   });
   if (st != ST_OK) return st;
 
@@ -777,16 +777,13 @@ ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, con
   ap.slot = slot;
   ap.L0 = (int32_t)L0;
   ap.T = n_tok;
-  const int64_t rows = (int64_t)n_tok * G;
-  const int n_tiles = (int)((rows + kMaxAttnRows - 1) / kMaxAttnRows);
   // algorithmic: main's KV once per (layer, head) + Q + O/LSE; flops: causal
   const double kv_bytes = (double)(L0 + n_tok) * c.n_kv_heads * c.head_dim * 2 * 2 * c.n_layers;
   const double io_bytes = (double)c.n_layers * n_tok * c.n_q_heads * (c.head_dim * 2 + c.head_dim * 4 + 4);
   const double keys = (double)n_tok * L0 + (double)n_tok * (n_tok + 1) / 2;
   const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
-  return run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s, [&] {
-    return launch_attend(P->kmap, P->vmap, ap, n_tiles, true, c.head_dim, s);
-  });
+  return run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
+                    [&] { return launch_merge_tc(P->kmap, P->vmap, ap, c.head_dim, s); });
 }
 
 ST_API st_status st_block_table(st_pool* P, st_seq seq, int32_t* out, int cap, int* n_pages,
