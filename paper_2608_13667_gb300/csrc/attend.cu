@@ -11,7 +11,7 @@
 // CTA layout (128 threads): warps 0..2 compute, warp 3 loads; 3 CTAs per SM.
 //   * Loader: reads page ids from the block table (32 at a time, one batch
 //     ahead) and issues one 2 KiB TMA tensor copy per (page, 64-wide half of
-//     the head, K|V) into a 2-stage ring of 4-page stages, signalling a
+//     the head, K|V) into a 4-stage ring of 2-page stages, signalling a
 //     per-stage mbarrier with the byte count.
 //   * Compute warp w owns query rows [16w, 16w+16).  Per stage it forms
 //     S = Q K^T on the tensor cores (mma.sync m16n8k16 bf16 -> fp32; K
@@ -34,8 +34,8 @@ namespace st {
 
 namespace {
 
-constexpr int kPPS = 4;            // pages per pipeline stage (64 keys)
-constexpr int kStages = 2;
+constexpr int kPPS = 2;            // pages per pipeline stage (32 keys)
+constexpr int kStages = 4;
 constexpr int kComputeWarps = 3;   // up to 48 stacked query rows
 constexpr int kThreads = (kComputeWarps + 1) * 32;
 constexpr float kLn2 = 0.69314718055994530942f;
