@@ -1,0 +1,489 @@
+// Paged attention on the 5th-generation tensor cores (tcgen05, accumulators
+// in tensor memory): fork-group decode partials and the merge prefill.
+//
+// Section 3.3 of the paper: every branch receives the snapshot H_t + R_t, so
+// the prefix KV is shared by all decoding streams; Section 4.4: branch load
+// is dominated by those cached-prefix reads.  A decode CTA owns one run of
+// pages of one KV head of one layer and stacks every query row that reads
+// it -- for a shared prefix all branches of the fork group x the G query
+// heads of the KV head (<= 48 rows) -- so each prefix page crosses HBM once
+// per group.  Section 3.5: the merged thoughts are appended after main's
+// context and read in order, so a merge CTA stacks 128 (thought row, head)
+// rows and walks main's pages up to its causal limit (row i sees keys
+// [0, L0 + i]).
+//
+// CTA layout (192 threads, 2 CTAs per SM):
+//   warps 0..3  softmax (only ceil(rows/32) of them run): thread r owns query
+//               row r = TMEM lane r.  It loads its Q row into shared memory;
+//               per stage it reads its scores from TMEM, masks keys past the
+//               run (and past its causal limit in the merge), keeps a running
+//               max that is raised only when a score exceeds it by more than
+//               2^8 (O in TMEM is then rescaled in place), and writes
+//               P = 2^(s - m) as bf16 over the stage's consumed K slot.  At the
+//               end it normalises O out of TMEM (decode: a split-KV partial
+//               with its log-sum-exp; merge: the final row).
+//   warp 4      loader: page ids from the block table (32 per read, one batch
+//               ahead), one 2 KiB TMA copy per (page, 64-wide half of D, K|V)
+//               into a ring of stages, per-stage mbarriers with byte counts.
+//   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M=128, N=64 keys)
+//               and O += P V (M=128, N=D) and commits them to mbarriers.  S is
+//               double-buffered in TMEM: S_{j+1} is issued before P_j V_j when
+//               its data has landed, so the softmax of stage j+1 overlaps the
+//               tensor work of stage j.
+//               A rescale of O first waits for the commit of P_{j-1} V_{j-1}.
+//
+// Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
+//   Q  [D/64][rows][64]       K-major A (SBO 1024)
+//   K  [D/64][keys][64]       K-major B (SBO 1024)
+//   P  [rows][keys]           K-major A (SBO 1024), written over K
+//   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
+// The MMA always computes 128 rows.  In decode only the first <= 48 Q and P
+// rows are written; rows past them read whatever follows in shared memory and
+// only produce accumulator rows that nobody reads (each output row depends
+// on its own A row only).  V rows of keys that are not valid (past the run,
+// or in pages a short last stage did not load) are zeroed before P V, so
+// stale shared or pool memory cannot turn 0 * x into NaN in a real row.
+#include <math.h>
+
+#include "kernels.cuh"
+#include "ptx.cuh"
+
+namespace st {
+
+namespace {
+
+constexpr int kMmaRows = 128;
+constexpr int kLoadWarp = 4, kMmaWarp = 5;
+constexpr int kThreads = 6 * 32;
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kTmemS = 0, kTmemO = 128;  // S buffers at 0 and 64
+constexpr float kRescaleThreshold = 8.f;  // log2 units
+constexpr float kLn2 = 0.69314718055994530942f;
+
+constexpr int cmax(int a, int b) { return a > b ? a : b; }
+
+template <int D, bool kDecode>
+struct TcCfg {
+  static constexpr int kHalves = D / 64;
+  static constexpr int kKeys = 64;                     // keys per stage
+  static constexpr int kPagesPerStage = kKeys / kPageTokens;
+  static constexpr int kStages = kDecode ? 3 : 2;
+  static constexpr int kQRows = kDecode ? 48 : 128;    // Q/P rows stored
+  static constexpr int kQHalfBytes = kQRows * 128;
+  static constexpr int kQBytes = kHalves * kQHalfBytes;
+  static constexpr int kKVHalfBytes = kKeys * 128;
+  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, kQRows * 128);  // K, then P
+  static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
+  static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
+  static constexpr int kRingBytes = kStages * kStageBytes;
+  // the MMA reads 128 rows of P from the last K slot: keep that inside the allocation
+  static constexpr int kOverread = cmax(0, kMmaRows * 128 - kStageBytes);
+  static constexpr int kBarOffset = kQBytes + kRingBytes + kOverread;
+  static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
+};
+
+template <int D, bool kDecode>
+__global__ void __launch_bounds__(kThreads, 2)
+    attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                     const AttnParams p) {
+  using C = TcCfg<D, kDecode>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
+  uint8_t* q_s = base;
+  uint8_t* ring = base + C::kQBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::kBarOffset);
+  uint64_t* full = bars;                 // [kStages]
+  uint64_t* empty = bars + C::kStages;   // [kStages]
+  uint64_t* s_full = bars + 2 * C::kStages;   // [2] per S buffer
+  uint64_t* p_full = s_full + 2;              // [2] per S buffer
+  uint64_t* o_ready = s_full + 4;             // one phase per P V
+  uint64_t* o_final = s_full + 5;
+  uint64_t* q_ready = s_full + 6;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 7);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int kvh = blockIdx.y;
+  const int layer = blockIdx.z;
+  const int G = p.G;
+
+  // ---- what this CTA reads and for whom ------------------------------------------
+  int slot, page_begin, n_pages, n_valid_keys, n_rows, min_limit, row_base = 0;
+  AttnItem item{};
+  if (kDecode) {
+    item = p.items[blockIdx.x];
+    slot = item.slot;
+    page_begin = item.page_begin;
+    n_pages = item.n_pages;
+    n_valid_keys = item.n_tokens;
+    n_rows = item.n_members * G;
+    min_limit = item.n_tokens;
+  } else {
+    slot = p.slot;
+    page_begin = 0;
+    row_base = blockIdx.x * kMmaRows;
+    n_rows = min(kMmaRows, p.T * G - row_base);
+    const int t_first = row_base / G;
+    const int t_last = (row_base + n_rows - 1) / G;
+    n_pages = (p.L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
+    n_valid_keys = p.L0 + p.T;
+    min_limit = p.L0 + t_first + 1;
+  }
+  const int n_tiles = (n_pages + C::kPagesPerStage - 1) / C::kPagesPerStage;
+  const int n_sw = (n_rows + 31) >> 5;   // softmax warps with rows
+  const int n_swt = n_sw * 32;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&p_full[b], n_swt);
+    }
+    mbar_init(o_ready, 1);
+    mbar_init(o_final, 1);
+    mbar_init(q_ready, n_swt);
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  // ---- loader --------------------------------------------------------------------
+  if (warp == kLoadWarp) {
+    if (lane == 0) {
+      prefetch_tensormap(&kmap);
+      prefetch_tensormap(&vmap);
+    }
+    // decode streams every page once; the merge's CTAs of one (layer, head)
+    // all walk the same pages
+    const uint64_t policy = kDecode ? l2_policy_evict_first() : l2_policy_evict_last();
+    const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
+    int base_id = 0;
+    int cur = lane < n_pages ? ids[lane] : 0;
+    int nxt = 32 + lane < n_pages ? ids[32 + lane] : 0;
+    int j = 0;
+    bool ok = true;
+    for (; j < n_tiles; ++j) {
+      const int s = j % C::kStages;
+      if (j >= C::kStages) {
+        int w = 1;
+        if (lane == 0) w = mbar_wait(&empty[s], ((j / C::kStages) - 1) & 1) ? 1 : 0;
+        w = __shfl_sync(0xffffffffu, w, 0);
+        if (!w) {
+          ok = false;
+          break;
+        }
+      }
+      const int page0 = j * C::kPagesPerStage;
+      if (page0 >= base_id + 32) {
+        base_id += 32;
+        cur = nxt;
+        nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
+      }
+      const int np = min(C::kPagesPerStage, n_pages - page0);
+      int blk[C::kPagesPerStage];
+#pragma unroll
+      for (int q = 0; q < C::kPagesPerStage; ++q)
+        blk[q] = __shfl_sync(0xffffffffu, cur, (page0 - base_id + q) & 31);
+      if (lane == 0) {
+        uint8_t* kst = ring + s * C::kStageBytes;
+        uint8_t* vst = kst + C::kKSlotBytes;
+        mbar_arrive_expect_tx(&full[s], (uint32_t)(np * 2 * C::kHalves * kPageTokens * 128));
+        for (int q = 0; q < np; ++q) {
+          int b = blk[q];
+          if ((uint64_t)b >= (uint64_t)p.n_blocks) {
+            atomicCAS(p.status, 0, kDevBadIndex);
+            b = 0;
+          }
+          const int c3 = layer * (int)p.n_blocks + b;
+#pragma unroll
+          for (int h = 0; h < C::kHalves; ++h) {
+            tma_load_4d(kst + h * C::kKVHalfBytes + q * kPageTokens * 128, &kmap, &full[s], 0, h,
+                        kvh * kPageTokens, c3, policy);
+            tma_load_4d(vst + h * C::kKVHalfBytes + q * kPageTokens * 128, &vmap, &full[s], 0, h,
+                        kvh * kPageTokens, c3, policy);
+          }
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      atomicCAS(p.status, 0, kDevTimeout);
+      for (int t = max(0, j - C::kStages); t < j; ++t) mbar_wait(&full[t % C::kStages], (t / C::kStages) & 1);
+    }
+    return;
+  }
+
+  // ---- MMA issuer ----------------------------------------------------------------
+  if (warp == kMmaWarp) {
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = tc_idesc_bf16(kMmaRows, C::kKeys, 0, 0);
+      constexpr uint32_t idesc_o = tc_idesc_bf16(kMmaRows, D, 0, 1);
+      const uint32_t q_addr = smem_addr(q_s);
+      bool ok = mbar_wait(q_ready, 0);
+      tc_fence_after_sync();
+      // S_j = Q K_j^T into S buffer j & 1
+      auto issue_s = [&](int j) -> bool {
+        const int s = j % C::kStages;
+        if (!mbar_wait(&full[s], (j / C::kStages) & 1)) return false;
+        tc_fence_after_sync();
+        const uint32_t k_addr = smem_addr(ring + s * C::kStageBytes);
+#pragma unroll
+        for (int h = 0; h < C::kHalves; ++h)
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16(tmem + kTmemS + (j & 1) * C::kKeys,
+                        tc_desc_sw128(q_addr + h * C::kQHalfBytes + kk * 32, 16, 1024),
+                        tc_desc_sw128(k_addr + h * C::kKVHalfBytes + kk * 32, 16, 1024), idesc_s,
+                        (h | kk) != 0);
+        tc_commit(&s_full[j & 1]);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        // S buffer (j+1)&1 was last read by the softmax of stage j-1, whose P
+        // this thread has already waited for.  Issue S_{j+1} ahead of P_j V_j
+        // only when its data has already landed, so that a slow load never
+        // delays P_j V_j.
+        const int jn = j + 1;
+        bool early = false;
+        if (jn < n_tiles && mbar_try_wait(&full[jn % C::kStages], (jn / C::kStages) & 1)) {
+          if (!issue_s(jn)) {
+            ok = false;
+            break;
+          }
+          early = true;
+        }
+        if (!mbar_wait(&p_full[j & 1], (j >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const int s = j % C::kStages;
+        const uint32_t k_addr = smem_addr(ring + s * C::kStageBytes);
+        const uint32_t v_addr = k_addr + C::kKSlotBytes;
+#pragma unroll
+        for (int ks = 0; ks < C::kKeys / 16; ++ks)
+          tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + ks * 32, 16, 1024),
+                      tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
+                      (j > 0 || ks > 0) ? 1u : 0u);
+        tc_commit(&empty[s]);
+        tc_commit(o_ready);
+        if (jn < n_tiles && !early && !issue_s(jn)) {
+          ok = false;
+          break;
+        }
+      }
+      tc_commit(o_final);
+      if (!ok) atomicCAS(p.status, 0, kDevTimeout);
+    }
+    __syncwarp();
+    named_barrier_sync(1, n_swt + 32);
+    tc_fence_after_sync();
+    tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
+  if (warp >= n_sw) return;
+
+  // ---- softmax warps ---------------------------------------------------------------
+  const int r = threadIdx.x;
+  const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
+  const bool valid = r < n_rows;
+  int qrow = 0, head = 0;
+  if (valid) {
+    if (kDecode) {
+      qrow = p.members[item.member_base + r / G];
+      head = kvh * G + r % G;
+    } else {
+      const int gr = row_base + r;
+      qrow = gr / G;
+      head = kvh * G + gr % G;
+    }
+  }
+  const int limit = (!kDecode && valid) ? p.L0 + qrow + 1 : n_valid_keys;
+  if (r < C::kQRows) {
+    const uint4* src = reinterpret_cast<const uint4*>(p.q + (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * D);
+#pragma unroll
+    for (int c = 0; c < D / 8; ++c) {
+      const uint4 v = valid ? src[c] : make_uint4(0u, 0u, 0u, 0u);
+      *reinterpret_cast<uint4*>(q_s + (c >> 3) * C::kQHalfBytes + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
+    }
+    fence_proxy_async_smem();
+  }
+  mbar_arrive(q_ready);
+
+  const float sl2 = p.scale_log2;
+  float m_used = -1e30f, l = 0.f;
+  bool ok = true;
+  for (int j = 0; j < n_tiles; ++j) {
+    const int s = j % C::kStages;
+    if (!__all_sync(0xffffffffu, mbar_wait(&s_full[j & 1], (j >> 1) & 1))) {
+      ok = false;
+      break;
+    }
+    tc_fence_after_sync();
+    float sc[C::kKeys];
+#pragma unroll
+    for (int c0 = 0; c0 < C::kKeys; c0 += 32) tmem_ld32(t_lane + kTmemS + (j & 1) * C::kKeys + c0, sc + c0);
+    const int key0 = j * C::kKeys;
+    const int np = min(C::kPagesPerStage, n_pages - j * C::kPagesPerStage);
+    const int loaded = np * kPageTokens;
+    const bool edge = key0 + C::kKeys > min_limit || loaded < C::kKeys;
+    float mx = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < C::kKeys; ++c) {
+      float x = sc[c] * sl2;
+      if (edge && (c >= loaded || key0 + c >= limit)) x = -INFINITY;
+      sc[c] = x;
+      mx = fmaxf(mx, x);
+    }
+    const float m_new = fmaxf(m_used, mx);
+    const bool need = valid && m_new > m_used + kRescaleThreshold;
+    if (__any_sync(0xffffffffu, need)) {
+      const float alpha = need ? ex2(m_used - m_new) : 1.f;
+      if (j > 0) {
+        // P_{j-1} V_{j-1} must have landed in O (P_j V_j cannot start before
+        // this thread's P_j, so the parity below is unambiguous)
+        if (!__all_sync(0xffffffffu, mbar_wait(o_ready, (j - 1) & 1))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+#pragma unroll 1
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          float o[32];
+          tmem_ld32(t_lane + kTmemO + c0, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tmem_st32(t_lane + kTmemO + c0, o);
+        }
+      }
+      l *= alpha;
+      if (need) m_used = m_new;
+    }
+    uint8_t* kslot = ring + s * C::kStageBytes;  // S_j has been consumed: P_j goes over K_j
+    if (valid) {
+      uint32_t pk[C::kKeys / 2];
+      float rs = 0.f;
+#pragma unroll
+      for (int c = 0; c < C::kKeys; c += 2) {
+        const float a = ex2(sc[c] - m_used), b = ex2(sc[c + 1] - m_used);
+        rs += a + b;
+        pk[c / 2] = pack_bf16(a, b);
+      }
+      l += rs;
+#pragma unroll
+      for (int c = 0; c < C::kKeys / 8; ++c)
+        *reinterpret_cast<uint4*>(kslot + r * 128 + ((c ^ (r & 7)) << 4)) =
+            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+    }
+    if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
+      // this stage's copies have landed (S_j was computed from them): zero
+      // the V rows of keys that are not valid
+      mbar_wait(&full[s], (j / C::kStages) & 1);
+      uint8_t* vslot = kslot + C::kKSlotBytes;
+      for (int t = r; t < C::kKeys * C::kHalves; t += n_swt) {
+        const int c = t % C::kKeys, h = t / C::kKeys;
+        if (c >= loaded || key0 + c >= n_valid_keys) {
+#pragma unroll
+          for (int x = 0; x < 8; ++x)
+            *reinterpret_cast<uint4*>(vslot + h * C::kKVHalfBytes + c * 128 + x * 16) = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before_sync();
+    mbar_arrive(&p_full[j & 1]);
+  }
+  if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0));
+  tc_fence_after_sync();
+  if (ok) {
+    const float inv = 1.f / l;
+    float* dst = nullptr;
+    float* dst_lse = nullptr;
+    if (valid) {
+      int64_t idx;
+      if (kDecode)
+        idx = (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * p.max_splits + item.split;
+      else
+        idx = ((int64_t)layer * p.T + qrow) * p.Hq + head;
+      dst = p.out_o + idx * D;
+      dst_lse = p.out_lse + idx;
+    }
+#pragma unroll 1
+    for (int c0 = 0; c0 < D; c0 += 32) {
+      float o[32];
+      tmem_ld32(t_lane + kTmemO + c0, o);
+      if (dst) {
+#pragma unroll
+        for (int i = 0; i < 32; i += 4)
+          *reinterpret_cast<float4*>(dst + c0 + i) =
+              make_float4(o[i] * inv, o[i + 1] * inv, o[i + 2] * inv, o[i + 3] * inv);
+      }
+    }
+    if (dst_lse) *dst_lse = (m_used + log2f(l)) * kLn2;
+  } else if (lane == 0) {
+    atomicCAS(p.status, 0, kDevTimeout);
+  }
+  tc_fence_before_sync();
+  named_barrier_sync(1, n_swt + 32);
+}
+
+template <int D, bool kDecode>
+cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_ctas,
+                        cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(attend_tc_kernel<D, kDecode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         TcCfg<D, kDecode>::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  dim3 grid(n_ctas, p.Hkv, p.L);
+  attend_tc_kernel<D, kDecode><<<grid, kThreads, TcCfg<D, kDecode>::kSmemBytes, s>>>(km, vm, p);
+  return cudaGetLastError();
+}
+
+template <int D>
+int decode_ctas_per_sm_t() {
+  if (cudaFuncSetAttribute(attend_tc_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           TcCfg<D, true>::kSmemBytes) != cudaSuccess)
+    return 0;
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, true>, kThreads,
+                                                    TcCfg<D, true>::kSmemBytes) != cudaSuccess)
+    return 0;
+  return n < 2 ? n : 2;  // two CTAs' TMEM (2 x 256 columns) fill an SM
+}
+
+}  // namespace
+
+cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_items,
+                             int D, cudaStream_t s) {
+  if (n_items <= 0) return cudaSuccess;
+  if (D == 128) return launch_tc_t<128, true>(km, vm, p, n_items, s);
+  if (D == 64) return launch_tc_t<64, true>(km, vm, p, n_items, s);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int D,
+                            cudaStream_t s) {
+  if (p.T <= 0) return cudaSuccess;
+  const int n_tiles = (p.T * p.G + kMmaRows - 1) / kMmaRows;
+  if (D == 128) return launch_tc_t<128, false>(km, vm, p, n_tiles, s);
+  if (D == 64) return launch_tc_t<64, false>(km, vm, p, n_tiles, s);
+  return cudaErrorInvalidValue;
+}
+
+int decode_tc_ctas_per_sm(int D) {
+  if (D == 128) return decode_ctas_per_sm_t<128>();
+  if (D == 64) return decode_ctas_per_sm_t<64>();
+  return 0;
+}
+
+}  // namespace st

@@ -1,0 +1,78 @@
+// Log-sum-exp combine of split-KV decode partials.
+//
+// A branch's decode is split into runs of pages (shared-prefix runs read for
+// the whole fork group, and the branch's own runs); each run yields a
+// normalised partial O_i with its log-sum-exp lse_i.  Since softmax over the
+// union of disjoint key sets is the lse-weighted mixture of the per-set
+// softmaxes, lse = log sum_i exp(lse_i) and O = sum_i exp(lse_i - lse) O_i.
+#include <math.h>
+
+#include "kernels.cuh"
+
+namespace st {
+
+namespace {
+
+// One warp per (layer, branch, query head): lse = log sum_i exp(lse_i),
+// O = sum_i exp(lse_i - lse) O_i over the branch's partials.
+template <int D>
+__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p) {
+  const int lane = threadIdx.x & 31;
+  const int64_t idx = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
+  if (idx >= total) return;
+  const int b = (int)((idx / p.Hq) % p.n_br);
+  const int ns = p.n_splits[b];
+  const float* lse_i = p.part_lse + idx * p.max_splits;
+  const float li = lane < ns ? lse_i[lane] : -INFINITY;
+  float mx = li;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  const float w = lane < ns ? expf(li - mx) : 0.f;
+  float sum = w;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  const float lse = mx + logf(sum);
+  constexpr int kPer = D / 32;
+  float out[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) out[e] = 0.f;
+  const float* po = p.part_o + idx * p.max_splits * D + lane * kPer;
+  for (int i = 0; i < ns; ++i) {
+    const float wi = __shfl_sync(0xffffffffu, w, i) / sum;
+    if (kPer == 4) {
+      const float4 x = *reinterpret_cast<const float4*>(po + (int64_t)i * D);
+      out[0] += wi * x.x;
+      out[1] += wi * x.y;
+      out[2] += wi * x.z;
+      out[3] += wi * x.w;
+    } else {
+      const float2 x = *reinterpret_cast<const float2*>(po + (int64_t)i * D);
+      out[0] += wi * x.x;
+      out[1] += wi * x.y;
+    }
+  }
+  float* dst = p.o + idx * D + lane * kPer;
+  if (kPer == 4)
+    *reinterpret_cast<float4*>(dst) = make_float4(out[0], out[1], out[2], out[3]);
+  else
+    *reinterpret_cast<float2*>(dst) = make_float2(out[0], out[1]);
+  if (lane == 0) p.lse[idx] = lse;
+}
+
+}  // namespace
+
+cudaError_t launch_combine(const CombineParams& p, int D, cudaStream_t s) {
+  const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
+  if (total == 0) return cudaSuccess;
+  const int grid = (int)((total + 3) / 4);
+  if (D == 128)
+    combine_kernel<128><<<grid, 128, 0, s>>>(p);
+  else if (D == 64)
+    combine_kernel<64><<<grid, 128, 0, s>>>(p);
+  else
+    return cudaErrorInvalidValue;
+  return cudaGetLastError();
+}
+
+}  // namespace st

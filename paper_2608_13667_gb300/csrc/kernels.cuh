@@ -2,9 +2,9 @@
 //
 //   table_update  -- refresh rows of the device block tables from the host's
 //   append_kv     -- copy-on-write page copies + scatter of new K/V rows
-//   attend        -- paged decode attention partials (mma.sync)
+//   attend_tc     -- paged decode partials and causal merge prefill
+//                    (tcgen05, TMEM accumulators)
 //   lse_combine   -- log-sum-exp combine of decode partials
-//   merge_tc      -- causal merge prefill (tcgen05, TMEM accumulators)
 #pragma once
 
 #include <cuda.h>
@@ -91,13 +91,14 @@ struct CombineParams {
 cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int32_t* values,
                                 int n_runs, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, int D, cudaStream_t s);
-cudaError_t launch_attend(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
-                          int n_ctas, int D, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, int D, cudaStream_t s);
+// Decode partials on tcgen05 (one CTA per item x KV head x layer).
+cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
+                             int n_items, int D, cudaStream_t s);
 // Causal merge prefill on tcgen05 (p.slot, p.L0, p.T, p.q -> p.out_o, p.out_lse).
 cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int D,
                             cudaStream_t s);
-// CTAs of the attend kernel resident per SM (0 on error).
-int attend_ctas_per_sm(int D);
+// CTAs of the tcgen05 decode kernel resident per SM (0 on error).
+int decode_tc_ctas_per_sm(int D);
 
 }  // namespace st

@@ -54,8 +54,8 @@ st_status setup_device(int dev) {
   if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return ST_ERR_CUDA;
   int sms = 0;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return ST_ERR_CUDA;
-  const int per_sm = attend_ctas_per_sm(128);
-  const int per_sm64 = attend_ctas_per_sm(64);
+  const int per_sm = decode_tc_ctas_per_sm(128);
+  const int per_sm64 = decode_tc_ctas_per_sm(64);
   if (per_sm < 1 || per_sm64 < 1) return ST_ERR_CUDA;
   g_sms[dev] = sms;
   g_ctas_per_sm[dev][1] = per_sm;
@@ -235,7 +235,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   ap.L = c.n_layers;
   ap.max_pages = table_stride;
   ap.max_splits = kSplitStride;
-  if (launch_attend(kmap, vmap, ap, n_items, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
+  if (launch_decode_tc(kmap, vmap, ap, n_items, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
   CombineParams cp{};
   cp.part_o = ap.out_o;
   cp.part_lse = ap.out_lse;

@@ -1,5 +1,6 @@
-// Inline-PTX helpers for sm_103a: mbarriers, TMA tensor loads, ldmatrix,
-// bf16 mma.sync and the exp2 unit.  Every wait here is bounded: it gives up
+// Inline-PTX helpers for sm_103a: mbarriers, TMA tensor loads, tcgen05
+// (MMA, TMEM alloc/load/store, commits, fences) and the exp2 unit.  Every
+// wait here is bounded: it gives up
 // after kWaitLimitNs of wall-clock time and reports failure to the caller,
 // which records ST_ERR_TIMEOUT in the device status word and winds down.
 #pragma once
@@ -88,33 +89,6 @@ __device__ __forceinline__ uint64_t l2_policy_evict_last() {
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr)
-               : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr)
-               : "memory");
-}
-
-// D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col).  A pure register
-// operation (not volatile), so the compiler may interleave independent MMAs.
-__device__ __forceinline__ void mma_bf16(float* c, uint32_t a0, uint32_t a1, uint32_t a2,
-                                         uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-      "{%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
 // Hardware base-2 exponential (MUFU.EX2; ex2(-inf) = +0).

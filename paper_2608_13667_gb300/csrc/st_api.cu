@@ -452,7 +452,7 @@ ST_API st_status st_pool_create(const st_config* cfg, void* k_pool, void* v_pool
   if (cudaMemset(P->ws, 0, P->lay.staging) != cudaSuccess) return bail(ST_ERR_CUDA);
   if (cudaDeviceGetAttribute(&P->sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
     return bail(ST_ERR_CUDA);
-  P->decode_ctas_per_sm = attend_ctas_per_sm(cfg->head_dim);
+  P->decode_ctas_per_sm = decode_tc_ctas_per_sm(cfg->head_dim);
   if (P->decode_ctas_per_sm < 1) return bail(ST_ERR_CUDA);
   if (cudaHostAlloc(reinterpret_cast<void**>(&P->h_stage), (size_t)kStageSlots * kStageSlotBytes,
                     cudaHostAllocDefault) != cudaSuccess)
@@ -718,7 +718,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.max_splits = c.max_splits;
   const int n_items = (int)items.size();
   st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
-    return launch_attend(P->kmap, P->vmap, ap, n_items, c.head_dim, s);
+    return launch_decode_tc(P->kmap, P->vmap, ap, n_items, c.head_dim, s);
   });
   if (st != ST_OK) return st;
 
