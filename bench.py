@@ -130,7 +130,7 @@ class ClockSampler:
 
 def _kernel_hash():
     h = hashlib.sha256()
-    for f in ("attend.cu", "ptx.cuh", "kernels.cuh"):
+    for f in ("attend_tc.cu", "ptx.cuh", "kernels.cuh"):
         with open(os.path.join(ROOT, "paper_2608_13667_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
