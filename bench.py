@@ -289,6 +289,52 @@ def run_ours(args, rank, ws, local):
     return res
 
 
+# --------------------------------------------------------------------------- profiling case
+
+def run_profile_small():
+    """A small case of both attention paths for ncu captures: the long-trajectory
+    decode with 4 layers (8.9 GB of KV per launch, beyond L2; three decode steps)
+    and one merge of 2048 thought rows onto a 16896-token main context (32 q /
+    8 kv heads, 4 layers).  Prints CUDA-event timings of the last decode and the
+    merge."""
+    import dataclasses
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import get, kv_rows, queries
+    dev = torch.device("cuda", 0)
+    st.build()
+    w = dataclasses.replace(get(4), n_layers=4)
+    pool, br = build_long_workload(w, dev)
+    n = len(br)
+    o = torch.empty((w.n_layers, n, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+    lse = torch.empty((w.n_layers, n, w.n_q_heads), dtype=torch.float32, device=dev)
+    pool.profile_enable(True)
+    for s in range(3):
+        k, v = kv_rows(w, ("step", s), n, device=dev)
+        shape = (w.n_layers, n, 1, w.n_kv_heads, w.head_dim)
+        pool.append_kv(br, k.view(shape), v.view(shape))
+        pool.decode_attn(br, queries(w, ("q", s), n, device=dev), o, lse)
+    pool.sync()
+    d = pool.profile_read()["decode_partial"]
+    w5 = dataclasses.replace(get(5), n_layers=4)
+    p5 = st.Pool(n_layers=4, n_q_heads=w5.n_q_heads, n_kv_heads=w5.n_kv_heads, head_dim=w5.head_dim,
+                 n_blocks=4096, seed=1, device=dev, max_seqs=8, max_pages=2048, max_decode_branches=8,
+                 max_splits=16)
+    m = p5.seq_create()
+    for c0 in range(0, 16896, 8448):
+        k, v = kv_rows(w5, ("ctx", c0), 8448, device=dev)
+        p5.append_kv([m], k.view(4, 1, 8448, 8, 128), v.view(4, 1, 8448, 8, 128))
+    k, v = kv_rows(w5, ("merge",), 2048, device=dev)
+    q = queries(w5, ("mq",), 2048, device=dev)
+    p5.profile_enable(True)
+    p5.merge(m, q, k, v)
+    p5.sync()
+    mg = p5.profile_read()["merge_prefill"]
+    print(json.dumps({"decode_ms_per_launch": d["total_ms"] / d["launches"],
+                      "decode_gbs": d["bytes"] / d["total_ms"] / 1e6,
+                      "merge_ms": mg["total_ms"], "merge_tflops": mg["flops"] / mg["total_ms"] / 1e9}))
+
+
 # --------------------------------------------------------------------------- oracle
 
 def oracle_sample_step(w, dev, layer, task=0):
@@ -361,7 +407,12 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-small", action="store_true",
+                    help="run the small decode + merge case used for ncu captures and exit")
     args = ap.parse_args()
+    if args.profile_small:
+        run_profile_small()
+        return
     rank, ws, local = _dist()
     if args.impl == "reference":
         res = run_reference(args, rank, ws, local)
