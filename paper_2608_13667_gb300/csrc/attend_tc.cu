@@ -327,22 +327,23 @@ __global__ void __launch_bounds__(kThreads, 2)
       break;
     }
     tc_fence_after_sync();
+    // raw scores q.k; the softmax works in the log2 domain, x = s * sl2
     float sc[C::kKeys];
-#pragma unroll
-    for (int c0 = 0; c0 < C::kKeys; c0 += 32) tmem_ld32(t_lane + kTmemS + (j & 1) * C::kKeys + c0, sc + c0);
+    static_assert(C::kKeys == 64, "one 64-column TMEM load per stage");
+    tmem_ld64(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
     const int key0 = j * C::kKeys;
     const int np = min(C::kPagesPerStage, n_pages - j * C::kPagesPerStage);
     const int loaded = np * kPageTokens;
     const bool edge = key0 + C::kKeys > min_limit || loaded < C::kKeys;
-    float mx = -INFINITY;
+    if (edge) {
 #pragma unroll
-    for (int c = 0; c < C::kKeys; ++c) {
-      float x = sc[c] * sl2;
-      if (edge && (c >= loaded || key0 + c >= limit)) x = -INFINITY;
-      sc[c] = x;
-      mx = fmaxf(mx, x);
+      for (int c = 0; c < C::kKeys; ++c)
+        if (c >= loaded || key0 + c >= limit) sc[c] = -INFINITY;
     }
-    const float m_new = fmaxf(m_used, mx);
+    float mx = sc[0];
+#pragma unroll
+    for (int c = 1; c < C::kKeys; ++c) mx = fmaxf(mx, sc[c]);
+    const float m_new = fmaxf(m_used, mx * sl2);  // sl2 > 0: max commutes with the scale
     const bool need = valid && m_new > m_used + kRescaleThreshold;
     if (__any_sync(0xffffffffu, need)) {
       const float alpha = need ? ex2(m_used - m_new) : 1.f;
@@ -372,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       float rs = 0.f;
 #pragma unroll
       for (int c = 0; c < C::kKeys; c += 2) {
-        const float a = ex2(sc[c] - m_used), b = ex2(sc[c + 1] - m_used);
+        const float a = ex2(fmaf(sc[c], sl2, -m_used)), b = ex2(fmaf(sc[c + 1], sl2, -m_used));
         rs += a + b;
         pk[c / 2] = pack_bf16(a, b);
       }
