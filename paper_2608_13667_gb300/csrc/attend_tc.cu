@@ -340,9 +340,14 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int c = 0; c < C::kKeys; ++c)
         if (c >= loaded || key0 + c >= limit) sc[c] = -INFINITY;
     }
-    float mx = sc[0];
+    // 8 independent max chains, then a tree (short dependency chains)
+    float mx8[8];
 #pragma unroll
-    for (int c = 1; c < C::kKeys; ++c) mx = fmaxf(mx, sc[c]);
+    for (int i = 0; i < 8; ++i) mx8[i] = sc[i];
+#pragma unroll
+    for (int c = 8; c < C::kKeys; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sc[c]);
+    const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                           fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
     const float m_new = fmaxf(m_used, mx * sl2);  // sl2 > 0: max commutes with the scale
     const bool need = valid && m_new > m_used + kRescaleThreshold;
     if (__any_sync(0xffffffffu, need)) {
@@ -370,14 +375,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint8_t* kslot = ring + s * C::kStageBytes;  // S_j has been consumed: P_j goes over K_j
     if (valid) {
       uint32_t pk[C::kKeys / 2];
-      float rs = 0.f;
+      float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < C::kKeys; c += 2) {
         const float a = ex2(fmaf(sc[c], sl2, -m_used)), b = ex2(fmaf(sc[c + 1], sl2, -m_used));
-        rs += a + b;
+        rs[(c >> 1) & 7] += a + b;
         pk[c / 2] = pack_bf16(a, b);
       }
-      l += rs;
+      l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
 #pragma unroll
       for (int c = 0; c < C::kKeys / 8; ++c)
         *reinterpret_cast<uint4*>(kslot + r * 128 + ((c ^ (r & 7)) << 4)) =
