@@ -148,6 +148,28 @@ ST_API st_status st_decode_attn(st_pool* pool, const st_seq* br, int n_br, const
 ST_API st_status st_merge(st_pool* pool, st_seq main, int n_tok, const void* q, const void* k,
                           const void* v, float* o, float* lse, void* stream);
 
+/* Thought harvest (Section 3.5): when the observation arrives, each branch's
+ * generated token stream is cut at its last closed </thought>.  Completed
+ * atoms (an open-tag token through the next close-tag token, tags included)
+ * are kept -- the first `cap` per branch (the paper caps at 5) -- an
+ * unfinished atom is dropped, a branch with no completed atom contributes
+ * nothing, and the kept atoms are concatenated in branch order.  An open tag
+ * inside an unfinished atom restarts it; a close tag outside an atom is
+ * ignored.  The count T written to *out_count is the number of thought rows
+ * to pass to st_merge (T = 0: nothing harvested, the turn is plain ReAct).
+ * streams:  device int32 [n_br][stride], token ids generated by each branch
+ * lens:     device int32 [n_br], tokens generated so far (clamped to stride)
+ * out_ids:  device int32 [n_br * stride], harvested ids (first T valid)
+ * out_src:  device int32 [n_br * stride] or NULL: b * stride + position of
+ *           each harvested token in its branch's stream
+ * out_atoms: device int32 [n_br] or NULL: atoms kept per branch
+ * out_count: device int32 [1]
+ * n_br <= 32, 0 <= cap <= 64, open_id != close_id.  Runs on `stream`; no pool
+ * is needed. */
+ST_API st_status st_harvest(const int32_t* streams, int stride, const int32_t* lens, int n_br,
+                            int32_t open_id, int32_t close_id, int cap, int32_t* out_ids,
+                            int32_t* out_src, int32_t* out_atoms, int32_t* out_count, void* stream);
+
 /* Release (Section 3.5: in-flight branches are cancelled and discarded):
  * drop one reference per table entry in logical order; pages reaching zero
  * go to the tail of the free list.  The handle becomes invalid. */

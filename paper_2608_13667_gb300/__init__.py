@@ -83,6 +83,7 @@ def lib():
         "st_sync": (I, [P, VP]),
         "st_profile_enable": (I, [P, I]),
         "st_profile_read": (I, [P, ctypes.POINTER(StKernelStat), I, ctypes.POINTER(I)]),
+        "st_harvest": (I, [VP, I, VP, I, ctypes.c_int32, ctypes.c_int32, I, VP, VP, VP, VP, VP]),
         "st_decode_attn_noalloc": (I, [ctypes.POINTER(StConfig), VP, VP, i32p, I, i32p, I, VP, VP, VP, VP]),
         "st_status_str": (ctypes.c_char_p, [I]),
         "st_last_error": (ctypes.c_char_p, [P]),
@@ -314,6 +315,32 @@ def st_release(pool, seq):
 
 def st_sync(pool, stream=None):
     return pool.sync(stream)
+
+
+def st_harvest(streams, lens, open_id, close_id, cap=5, stream=None):
+    """Thought harvest on the device (see include/st.h).  streams: int32
+    [n_br, stride] CUDA tensor of generated token ids; lens: int32 [n_br] CUDA
+    tensor.  Returns (ids [T], src [T], atoms [n_br]) as CUDA tensors; T is read
+    back to the host to size the result."""
+    import torch
+    n_br, stride = streams.shape
+    for t, name in ((streams, "streams"), (lens, "lens")):
+        if t.dtype != torch.int32 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous int32 CUDA tensor")
+    out_ids = torch.empty(n_br * stride, dtype=torch.int32, device=streams.device)
+    out_src = torch.empty_like(out_ids)
+    atoms = torch.empty(n_br, dtype=torch.int32, device=streams.device)
+    count = torch.empty(1, dtype=torch.int32, device=streams.device)
+    if stream is None:
+        stream = torch.cuda.current_stream(streams.device)
+    st = lib().st_harvest(ctypes.c_void_p(streams.data_ptr()), stride, ctypes.c_void_p(lens.data_ptr()), n_br,
+                          int(open_id), int(close_id), cap, ctypes.c_void_p(out_ids.data_ptr()),
+                          ctypes.c_void_p(out_src.data_ptr()), ctypes.c_void_p(atoms.data_ptr()),
+                          ctypes.c_void_p(count.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+    if st != ST_OK:
+        raise STError(st, "st_harvest: " + lib().st_status_str(st).decode())
+    T = int(count.item())
+    return out_ids[:T], out_src[:T], atoms
 
 
 def st_decode_attn_noalloc(geom, k_pool, v_pool, page_tables, seq_len, q, o, lse, stream=None):
