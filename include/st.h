@@ -111,6 +111,15 @@ ST_API st_status st_seq_create(st_pool* pool, st_seq* out);
  * free.  out_aux receives n_aux handles. */
 ST_API st_status st_fork(st_pool* pool, st_seq seq, int n_aux, st_seq* out_aux);
 
+/* Fork from an earlier point of `seq` (Table 2 of the paper: "w/o R_t" forks
+ * before the just-finished thought, "fork onset" at the start of the turn):
+ * the n_aux children see only seq's first `length` rows (0 <= length <=
+ * seq's length).  They take the first ceil(length / page) table entries with
+ * one reference each; a child's last page may still hold seq's rows past
+ * `length`, which the child's first append copies away (copy-on-write of
+ * rows [0, length % page)).  Otherwise as st_fork. */
+ST_API st_status st_fork_at(st_pool* pool, st_seq seq, int64_t length, int n_aux, st_seq* out_aux);
+
 /* Append n_tok KV rows to each of the n_br sequences in br (in that order;
  * each sequence at most once per call).
  * k, v: device bf16 [n_layers][n_br][n_tok][n_kv_heads][head_dim].

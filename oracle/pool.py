@@ -17,7 +17,11 @@ project's reading, and the CUDA library must reproduce them bit-exactly:
   at the copy.  A page with refcount 1 is written in place.
 * Fork copies the parent's table and takes one reference on every entry; it
   allocates no page.  It fails without any change if fewer than n_aux
-  sequence slots are free.
+  sequence slots are free.  A fork at an earlier point (Table 2's "w/o R_t"
+  and "fork onset": the branches see only the first `length` rows of the
+  parent) copies the first ceil(length / page) entries; the child's last page
+  may then hold parent rows past the child's length, which the child's first
+  append copies away like any shared partial page.
 * Release drops one reference per table entry in logical order; pages that
   reach zero are pushed to the FIFO tail in that order.
 * A multi-branch append processes branches in the order given; it fails
@@ -122,6 +126,23 @@ class RefPool:
             s = Seq()
             s.table = list(src.table)
             s.length = src.length
+            for b in s.table:
+                self.ref[b] += 1
+            self.seqs.append(s)
+            out.append(len(self.seqs) - 1)
+        return out
+
+    def fork_at(self, parent, length, n_aux):
+        src = self.seqs[parent]
+        assert src.alive and 0 <= length <= src.length
+        if len(self.live()) + n_aux > self.max_seqs:
+            raise OutOfSlots()
+        out = []
+        n_pages = -(-length // self.page)
+        for _ in range(n_aux):
+            s = Seq()
+            s.table = list(src.table[:n_pages])
+            s.length = length
             for b in s.table:
                 self.ref[b] += 1
             self.seqs.append(s)

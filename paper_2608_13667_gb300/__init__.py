@@ -73,6 +73,7 @@ def lib():
         "st_pool_destroy": (I, [P]),
         "st_seq_create": (I, [P, i64p]),
         "st_fork": (I, [P, I64, I, i64p]),
+        "st_fork_at": (I, [P, I64, I64, I, i64p]),
         "st_append_kv": (I, [P, i64p, I, I, VP, VP, VP]),
         "st_decode_attn": (I, [P, i64p, I, VP, VP, VP, VP]),
         "st_merge": (I, [P, I64, I, VP, VP, VP, VP, VP, VP]),
@@ -193,6 +194,11 @@ class Pool:
         self._check(lib().st_fork(self._h, int(seq), n_aux, out), "st_fork")
         return [out[i] for i in range(n_aux)]
 
+    def fork_at(self, seq, length, n_aux=4):
+        out = (ctypes.c_int64 * max(1, n_aux))()
+        self._check(lib().st_fork_at(self._h, int(seq), int(length), n_aux, out), "st_fork_at")
+        return [out[i] for i in range(n_aux)]
+
     def append_kv(self, branches, k, v, stream=None):
         """k, v: bf16 [L][n_br][n_tok][Hkv][D] (a metadata-only pool takes
         k = v = None and n_tok passed as an int in k's place)."""
@@ -295,6 +301,10 @@ def st_seq_create(pool):
 
 def st_fork(pool, seq, n_aux=4):
     return pool.fork(seq, n_aux)
+
+
+def st_fork_at(pool, seq, length, n_aux=4):
+    return pool.fork_at(seq, length, n_aux)
 
 
 def st_append_kv(pool, branches, k, v, stream=None):

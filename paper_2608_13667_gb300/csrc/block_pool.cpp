@@ -69,17 +69,22 @@ int BlockPool::create_seq() {
 }
 
 bool BlockPool::fork(int parent, int n_aux, int* out) {
+  return fork_at(parent, slots_[parent].len, n_aux, out);
+}
+
+bool BlockPool::fork_at(int parent, int64_t length, int n_aux, int* out) {
   int found = 0;
   for (int i = 0; i < (int)slots_.size() && found < n_aux; ++i)
     if (!slots_[i].live) out[found++] = i;
   if (found < n_aux) return false;
   const SeqSlot& src = slots_[parent];
+  const size_t n_pages = (size_t)((length + page_ - 1) / page_);
   for (int a = 0; a < n_aux; ++a) {
     SeqSlot& s = slots_[out[a]];
     s.live = true;
     s.family = src.family;
-    s.len = src.len;
-    s.table = src.table;
+    s.len = length;
+    s.table.assign(src.table.begin(), src.table.begin() + n_pages);
     s.dirty_lo = s.dirty_hi = 0;
     s.mark_dirty(0, (int32_t)s.table.size());
     for (int32_t b : s.table) ++ref_[b];

@@ -55,6 +55,9 @@ class BlockPool {
   int create_seq();
   // Fills out[n_aux] with new slots; false (no change) when slots run out.
   bool fork(int parent, int n_aux, int* out);
+  // Fork from the parent's first `length` rows (0 <= length <= parent length):
+  // the children take the first ceil(length / page) table entries.
+  bool fork_at(int parent, int64_t length, int n_aux, int* out);
   // Pages an append of n_tok rows to `slot` takes from the free list.
   int64_t pages_needed(int slot, int64_t n_tok) const;
   // Would the table outgrow max_pages?

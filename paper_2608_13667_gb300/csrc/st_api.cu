@@ -520,10 +520,20 @@ ST_API st_status st_fork(st_pool* P, st_seq seq, int n_aux, st_seq* out_aux) {
   if (!P) return ST_ERR_INVALID;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+  return st_fork_at(P, seq, P->pool->slot(slot).len, n_aux, out_aux);
+}
+
+ST_API st_status st_fork_at(st_pool* P, st_seq seq, int64_t length, int n_aux, st_seq* out_aux) {
+  if (!P) return ST_ERR_INVALID;
+  int slot;
+  if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
   if (n_aux < 0 || (n_aux > 0 && !out_aux)) return fail(P, ST_ERR_INVALID, "bad n_aux/out_aux");
+  if (length < 0 || length > P->pool->slot(slot).len)
+    return fail(P, ST_ERR_INVALID, "fork point %lld outside [0, %lld]", (long long)length,
+                (long long)P->pool->slot(slot).len);
   if (n_aux == 0) return ST_OK;
   std::vector<int> slots(n_aux);
-  if (!P->pool->fork(slot, n_aux, slots.data()))
+  if (!P->pool->fork_at(slot, length, n_aux, slots.data()))
     return fail(P, ST_ERR_OOM, "fewer than %d free sequence slots", n_aux);
   for (int i = 0; i < n_aux; ++i) out_aux[i] = make_handle(P, slots[i]);
   return ST_OK;

@@ -53,6 +53,20 @@ class Run:
             self.hist[k] = list(self.hist[rid])
         return kids
 
+    def fork_at(self, rid, length, n_aux=4):
+        kids = self.ref.fork_at(rid, length, n_aux)
+        cut, left = [], length
+        for tag, off, cnt in self.hist[rid]:
+            if left <= 0:
+                break
+            take = min(cnt, left)
+            cut.append((tag, off, take))
+            left -= take
+        for k, h in zip(kids, self.pool.fork_at(self.handle[rid], length, n_aux)):
+            self.handle[k] = h
+            self.hist[k] = list(cut)
+        return kids
+
     def append(self, rids, n_tok, tag):
         w = self.w
         n = len(rids)

@@ -299,3 +299,30 @@ def test_merge_of_nothing_changes_nothing(stlib):
     run.pool.merge(run.handle[m], e, kv, kv)
     assert snap == (run.pool.refcounts(), run.pool.free_list(), run.pool.block_table(run.handle[m]))
     run.pool.sync()
+
+
+@pytest.mark.parametrize("variant", ["without_r_t", "fork_onset"])
+def test_fork_point_variants(stlib, variant):
+    """Table 2 of the paper: branches that do not see the just-finished
+    thought R_t ("w/o R_t": fork at the end of H_t) or fork when the turn
+    starts ("fork onset": the window also covers the Thought phase, so the
+    branches decode while main is still writing R_t)."""
+    w = _small(128, 32, 8, n_blocks=512, L=2)
+    run = Run(w, max_seqs=8, max_decode_branches=8, max_splits=8)
+    m = run.create()
+    run.append([m], 1003, ("H_t",))                     # history, ends mid-page
+    if variant == "without_r_t":
+        run.append([m], 77, ("R_t",))                   # main's thought
+        aux = run.fork_at(m, 1003, 4)                   # branches see H_t only
+    else:
+        aux = run.fork(m, 4)                            # fork at turn onset
+        run.append([m], 77, ("R_t",))                   # main thinks while branches run
+    for step in range(20):
+        run.append([m] + aux, 1, ("step", step))
+        q, o, lse = run.decode([m] + aux, ("q", step))
+        if step in (0, 19):
+            for layer in range(2):
+                o_ref, l_ref = run.oracle_decode([m] + aux, q, layer)
+                compare(o[layer], lse[layer], o_ref, l_ref, f"{variant} step {step} layer {layer}")
+    run.pool.sync()
+    run.check_tables()

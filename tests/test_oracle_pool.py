@@ -69,10 +69,15 @@ def test_random_operation_sequences_keep_invariants_and_content():
                     pool.append(ids, n, labels)
                     for i, lab in zip(ids, labels):
                         history[i] += lab
-                elif op < 0.65 and live:
+                elif op < 0.58 and live:
                     parent = r.choice(live)
                     for c in pool.fork(parent, r.randint(1, 4)):
                         history[c] = list(history[parent])
+                elif op < 0.65 and live:
+                    parent = r.choice(live)
+                    cut = r.randint(0, pool.seqs[parent].length)
+                    for c in pool.fork_at(parent, cut, r.randint(1, 3)):
+                        history[c] = list(history[parent][:cut])
                 elif op < 0.85 and len(live) > 1:
                     pool.release(r.choice(live))
                 else:
@@ -166,3 +171,25 @@ def test_merge_is_an_append_to_main():
     p1.merge(0, 50)
     p2.append([0], 50)
     assert p1.seqs[0].table == p2.seqs[0].table and list(p1.free) == list(p2.free)
+
+
+def test_fork_at_full_length_is_fork():
+    p1, p2 = P.RefPool(64, 5), P.RefPool(64, 5)
+    for p in (p1, p2):
+        p.create()
+        p.append([0], 37)
+    a = p1.fork(0, 2)
+    b = p2.fork_at(0, 37, 2)
+    assert [p1.seqs[i].table for i in a] == [p2.seqs[i].table for i in b] and p1.ref == p2.ref
+
+
+def test_fork_at_mid_page_copies_on_first_append():
+    pool = P.RefPool(32, 6, track_content=True)
+    m = pool.create()
+    pool.append([m], 40, [[("m", i) for i in range(40)]])
+    (c,) = pool.fork_at(m, 21, 1)                 # page 1 holds rows 16..31 of main; the child sees 16..20
+    assert pool.seqs[c].table == pool.seqs[m].table[:2]
+    ev = pool.append([c], 1, [[("c", 0)]])
+    assert len(ev) == 1 and ev[0][0] == pool.seqs[m].table[1] and ev[0][2] == 5
+    assert pool.read(c) == [("m", i) for i in range(21)] + [("c", 0)]
+    assert pool.read(m) == [("m", i) for i in range(40)]

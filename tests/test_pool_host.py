@@ -52,14 +52,17 @@ def test_random_traces_match_reference_bit_exactly(stlib, seed):
         elif op < 0.65 and live:
             parent = r.choice(live)
             n_aux = r.randint(1, 4)
+            at = r.random() < 0.4
+            cut = r.randint(0, ref.seqs[parent].length)
             try:
-                kids = ref.fork(parent, n_aux)
+                kids = ref.fork_at(parent, cut, n_aux) if at else ref.fork(parent, n_aux)
             except R.OutOfSlots:
                 with pytest.raises(stlib.STError) as e:
-                    lp.fork(handles[parent], n_aux)
+                    lp.fork_at(handles[parent], cut, n_aux) if at else lp.fork(handles[parent], n_aux)
                 assert e.value.status == stlib.ST_ERR_OOM
             else:
-                for k, h in zip(kids, lp.fork(handles[parent], n_aux)):
+                new = lp.fork_at(handles[parent], cut, n_aux) if at else lp.fork(handles[parent], n_aux)
+                for k, h in zip(kids, new):
                     handles[k] = h
         elif op < 0.75 and live:
             m = r.choice(live)
@@ -186,3 +189,15 @@ def test_metadata_pool_refuses_attention(stlib):
     arr = (ctypes.c_int64 * 1)(a)
     st = L.st_decode_attn(lp._h, arr, 1, ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), None)
     assert st == stlib.ST_ERR_STATE
+
+
+def test_fork_at_rejects_points_past_the_end(stlib):
+    lp = _meta(stlib, 16, 0)
+    a = lp.seq_create()
+    lp.append_kv([a], 20, None)
+    for bad in (-1, 21):
+        with pytest.raises(stlib.STError) as e:
+            lp.fork_at(a, bad, 1)
+        assert e.value.status == stlib.ST_ERR_INVALID
+    (c,) = lp.fork_at(a, 0, 1)
+    assert lp.block_table(c) == ([], 0)
