@@ -57,6 +57,13 @@ typedef enum {
 } st_status;
 
 typedef int64_t st_seq;
+
+/* Test hook for the device-timeout path: with this flag the decode kernel's
+ * loader issues no copies, so its bounded waits (2 s) run out, the kernel
+ * records ST_ERR_TIMEOUT in the device status word and returns without
+ * faulting, and the next st_sync reports ST_ERR_TIMEOUT.  Outputs of such a
+ * call are undefined.  Never set in normal use. */
+#define ST_FLAG_HOLD_LOADS 1
 typedef struct st_pool st_pool;
 
 /* Pool geometry and capacities.
@@ -73,7 +80,7 @@ typedef struct {
   int32_t max_pages;           /* block-table capacity per sequence, in pages */
   int32_t max_decode_branches; /* branches per st_decode_attn call */
   int32_t max_splits;          /* partial results per (branch, head, layer) in one decode; 2..32 */
-  int32_t reserved;
+  int32_t flags;               /* ST_FLAG_* bits; 0 for normal use */
   int64_t n_blocks;            /* physical pages in the pool (each spans all layers and KV heads) */
   uint64_t seed;               /* seeds the free-list shuffle (splitmix64, Fisher-Yates) */
 } st_config;

@@ -16,6 +16,7 @@ import os
 from ._build import LIB, build  # noqa: F401
 
 ST_OK, ST_ERR_INVALID, ST_ERR_OOM, ST_ERR_STATE, ST_ERR_CUDA, ST_ERR_TIMEOUT = range(6)
+ST_FLAG_HOLD_LOADS = 1
 PAGE = 16
 
 
@@ -36,7 +37,7 @@ class StConfig(ctypes.Structure):
         ("max_pages", ctypes.c_int32),
         ("max_decode_branches", ctypes.c_int32),
         ("max_splits", ctypes.c_int32),
-        ("reserved", ctypes.c_int32),
+        ("flags", ctypes.c_int32),
         ("n_blocks", ctypes.c_int64),
         ("seed", ctypes.c_uint64),
     ]
@@ -111,12 +112,12 @@ class Pool:
 
     def __init__(self, n_layers, n_q_heads, n_kv_heads, head_dim, n_blocks, seed=0,
                  max_seqs=64, max_pages=None, max_decode_branches=16, max_splits=16,
-                 device="cuda"):
+                 device="cuda", flags=0):
         self.cfg = StConfig(
             n_layers=n_layers, n_q_heads=n_q_heads, n_kv_heads=n_kv_heads, head_dim=head_dim,
             page_size=PAGE, max_seqs=max_seqs,
             max_pages=int(max_pages if max_pages is not None else n_blocks),
-            max_decode_branches=max_decode_branches, max_splits=max_splits, reserved=0,
+            max_decode_branches=max_decode_branches, max_splits=max_splits, flags=flags,
             n_blocks=n_blocks, seed=seed)
         L = lib()
         self._h = ctypes.c_void_p()

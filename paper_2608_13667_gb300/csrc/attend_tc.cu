@@ -156,6 +156,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 
   // ---- loader --------------------------------------------------------------------
   if (warp == kLoadWarp) {
+    if (p.hold_loads) return;  // test hook: nothing arrives, the other roles' waits run out
     if (lane == 0) {
       prefetch_tensormap(&kmap);
       prefetch_tensormap(&vmap);

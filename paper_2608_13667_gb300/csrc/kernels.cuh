@@ -77,6 +77,7 @@ struct AttnParams {
   int32_t n_rows_q;        // decode: n_br; merge: T
   int32_t Hq, Hkv, G, L, max_pages, max_splits;
   int32_t slot, L0, T;     // merge only: main's slot, length before the append, thought rows
+  int32_t hold_loads;      // test hook (ST_FLAG_HOLD_LOADS): the loader issues nothing
 };
 
 struct CombineParams {

@@ -726,6 +726,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.L = c.n_layers;
   ap.max_pages = c.max_pages;
   ap.max_splits = c.max_splits;
+  ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
   const int n_items = (int)items.size();
   st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
     return launch_decode_tc(P->kmap, P->vmap, ap, n_items, c.head_dim, s);

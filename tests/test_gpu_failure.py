@@ -1,0 +1,41 @@
+"""The device-timeout path: every wait in the attention kernel is bounded.
+With the ST_FLAG_HOLD_LOADS test hook nothing ever arrives on the decode's
+stage barriers; the waits run out (2 s), the kernel records ST_ERR_TIMEOUT
+and returns without faulting, st_sync reports it, and the context stays
+usable for a normal pool afterwards."""
+import time
+
+import pytest
+import torch
+
+import paper_2608_13667_gb300 as stpkg
+from fg_harness import Run, compare
+from workloads import Workload, kv_rows, queries
+
+pytestmark = pytest.mark.gpu
+
+
+def test_decode_wait_runs_out_and_is_reported(stlib):
+    w = Workload(name="hold", n_layers=1, n_q_heads=8, n_kv_heads=1, head_dim=128, n_blocks=16, seed=41)
+    pool = stpkg.Pool(n_layers=1, n_q_heads=8, n_kv_heads=1, head_dim=128, n_blocks=16, seed=41,
+                      max_seqs=2, max_decode_branches=1, max_splits=2, flags=stpkg.ST_FLAG_HOLD_LOADS)
+    a = pool.seq_create()
+    k, v = kv_rows(w, ("ctx",), 20, device="cuda")
+    pool.append_kv([a], k.view(1, 1, 20, 1, 128), v.view(1, 1, 20, 1, 128))
+    q = queries(w, ("q",), 1, device="cuda")
+    t0 = time.time()
+    pool.decode_attn([a], q)                 # one CTA: its waits run out after ~2 s
+    with pytest.raises(stpkg.STError) as e:
+        pool.sync()
+    assert e.value.status == stpkg.ST_ERR_TIMEOUT
+    assert time.time() - t0 < 60
+    pool.sync()                              # the status word was cleared
+    pool.close()
+    # the context is still usable
+    run = Run(w, max_seqs=2, max_decode_branches=1, max_splits=2)
+    b = run.create()
+    run.append([b], 20, ("ctx2",))
+    q2, o, lse = run.decode([b], ("q2",))
+    run.pool.sync()
+    o_ref, l_ref = run.oracle_decode([b], q2, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "after timeout")
