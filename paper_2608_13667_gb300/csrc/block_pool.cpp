@@ -111,20 +111,20 @@ void BlockPool::append(const int* slots, int n, int64_t n_tok, std::vector<CowEv
   for (int i = 0; i < n; ++i) {
     SeqSlot& s = slots_[slots[i]];
     const int64_t off = s.len % page_;
-    const int32_t first_dirty = (int32_t)(s.len / page_);
     if (off != 0 && ref_[s.table.back()] > 1) {
       const int32_t old = s.table.back();
       const int32_t fresh = pop_free();
       --ref_[old];
       s.table.back() = fresh;
       cows->push_back(CowEvent{old, fresh, (int32_t)off});
+      s.mark_dirty((int32_t)s.table.size() - 1, (int32_t)s.table.size());
     }
     const int64_t new_len = s.len + n_tok;
     const int64_t have = (int64_t)s.table.size();
     const int64_t want = (new_len + page_ - 1) / page_;
     for (int64_t pg = have; pg < want; ++pg) s.table.push_back(pop_free());
     s.len = new_len;
-    s.mark_dirty(first_dirty, (int32_t)s.table.size());
+    s.mark_dirty((int32_t)have, (int32_t)s.table.size());  // only entries that changed
   }
 }
 

@@ -183,7 +183,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   int64_t chunk = std::max<int64_t>(16, ((units + target - 1) / target + 3) / 4 * 4);
   for (int gi = 0; gi < n_groups; ++gi) {
     const Grp& g = groups[gi];
-    const int32_t k = (int32_t)std::min<int64_t>(kSplitStride / 2, (g.pages + chunk - 1) / chunk);
+    const int32_t k = (int32_t)std::min<int64_t>(kSplitStride - 2, (g.pages + chunk - 1) / chunk);
     const int32_t mbase = n_members;
     for (int m = 0; m < g.count; ++m) plan.members[n_members++] = g.mem[m];
     for (int32_t ci = 0; ci < k; ++ci) {

@@ -57,7 +57,7 @@ def _single_turn():
         name="single_agent_turn", n_layers=1, n_q_heads=32, n_kv_heads=8, head_dim=128,
         n_blocks=1024, seed=1, n_tasks=1, prefix=(8192,),
         suffix=((256, 256, 256, 256, 256),), steps=256,
-        limits=dict(max_seqs=8, max_decode_branches=5, max_splits=16, max_pages=1024))
+        limits=dict(max_seqs=8, max_decode_branches=5, max_splits=32, max_pages=1024))
 
 
 def _batched():
