@@ -335,6 +335,76 @@ def run_profile_small():
                       "merge_ms": mg["total_ms"], "merge_tflops": mg["flops"] / mg["total_ms"] / 1e9}))
 
 
+def run_cycle():
+    """The full fork / decode / merge cycle (8 tasks x 16384-token contexts,
+    32 layers, 32/8 heads): per turn, fork 4 branches per task, 512 steps in
+    which main + branches + 64 unforked 2048-token sequences append one row
+    and decode, merge 2048 thought rows into each main, release.  5 turns.
+    Prints the time of the whole cycle and of its decode and merge parts."""
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import get, kv_rows, queries
+    w = get(5)
+    dev = torch.device("cuda", 0)
+    st.build()
+    pool = st.Pool(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads, head_dim=w.head_dim,
+                   n_blocks=w.n_blocks, seed=w.seed, device=dev, **w.limits)
+    L, Hkv, D = w.n_layers, w.n_kv_heads, w.head_dim
+    mains = []
+    for t in range(w.n_tasks):
+        m = pool.seq_create()
+        for c0 in range(0, w.prefix[t], PREFIX_CHUNK):
+            n = min(PREFIX_CHUNK, w.prefix[t] - c0)
+            k, v = kv_rows(w, ("prefix", t, c0), n, device=dev)
+            pool.append_kv([m], k.view(L, 1, n, Hkv, D), v.view(L, 1, n, Hkv, D))
+        mains.append(m)
+    n_rows = w.n_tasks * (w.n_aux + 1) + w.singletons
+    # step inputs drawn once and reused (values do not change the work)
+    sk, sv = kv_rows(w, ("step",), n_rows, device=dev)
+    sk, sv = sk.view(L, n_rows, 1, Hkv, D), sv.view(L, n_rows, 1, Hkv, D)
+    sq = queries(w, ("q",), n_rows, device=dev)
+    mk, mv = kv_rows(w, ("merge",), w.merge_tokens, device=dev)
+    mq = queries(w, ("mq",), w.merge_tokens, device=dev)
+    o = torch.empty((L, n_rows, w.n_q_heads, D), dtype=torch.float32, device=dev)
+    lse = torch.empty((L, n_rows, w.n_q_heads), dtype=torch.float32, device=dev)
+    mo = torch.empty((L, w.merge_tokens, w.n_q_heads, D), dtype=torch.float32, device=dev)
+    ml = torch.empty((L, w.merge_tokens, w.n_q_heads), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize(dev)
+    pool.profile_enable(True)
+    t_all = time.perf_counter()
+    for turn in range(w.turns):
+        singles = [pool.seq_create() for _ in range(w.singletons)]
+        for i in range(0, w.singletons, 8):
+            k, v = kv_rows(w, ("single", turn, i), 8 * w.singleton_len, device=dev)
+            pool.append_kv(singles[i:i + 8], k.view(L, 8, w.singleton_len, Hkv, D),
+                           v.view(L, 8, w.singleton_len, Hkv, D))
+        groups = [[m] + pool.fork(m, w.n_aux) for m in mains]
+        rids = [r for g in groups for r in g] + singles
+        for step in range(w.steps):
+            pool.append_kv(rids, sk, sv)
+            pool.decode_attn(rids, sq, o, lse)
+        for m in mains:
+            pool.merge(m, mq, mk, mv, mo, ml)
+        for g in groups:
+            for a in g[1:]:
+                pool.release(a)
+        for s_ in singles:
+            pool.release(s_)
+    torch.cuda.synchronize(dev)
+    total = time.perf_counter() - t_all
+    pool.sync()
+    stats = pool.profile_read()
+    dec, mer = stats["decode_partial"], stats["merge_prefill"]
+    print(json.dumps({
+        "workload": w.name, "seconds": total,
+        "decode_steps": dec["launches"], "decode_ms_per_step": dec["total_ms"] / dec["launches"],
+        "decode_gbs": dec["bytes"] / dec["total_ms"] / 1e6,
+        "branch_steps_per_s": dec["launches"] * n_rows / total,
+        "merges": mer["launches"], "merge_ms": mer["total_ms"] / mer["launches"],
+        "merge_tflops": mer["flops"] / mer["total_ms"] / 1e9,
+        "kernels": {k: {"launches": v["launches"], "ms": v["total_ms"]} for k, v in stats.items() if v["launches"]}}))
+
+
 # --------------------------------------------------------------------------- oracle
 
 def oracle_sample_step(w, dev, layer, task=0):
@@ -409,9 +479,14 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-small", action="store_true",
                     help="run the small decode + merge case used for ncu captures and exit")
+    ap.add_argument("--cycle", action="store_true",
+                    help="time the full fork/decode/merge cycle workload and exit")
     args = ap.parse_args()
     if args.profile_small:
         run_profile_small()
+        return
+    if args.cycle:
+        run_cycle()
         return
     rank, ws, local = _dist()
     if args.impl == "reference":

@@ -59,6 +59,7 @@ constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kTmemS = 0, kTmemO = 128;  // S buffers at 0 and 64
 constexpr float kRescaleThreshold = 8.f;  // log2 units
 constexpr float kLn2 = 0.69314718055994530942f;
+constexpr int kMaxDevices = 64;
 
 constexpr int cmax(int a, int b) { return a > b ? a : b; }
 
@@ -444,12 +445,17 @@ __global__ void __launch_bounds__(kThreads, 2)
 template <int D, bool kDecode>
 cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_ctas,
                         cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attend_tc_kernel<D, kDecode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         TcCfg<D, kDecode>::kSmemBytes);
+  // the shared-memory opt-in is a per-device function attribute
+  static bool configured[kMaxDevices] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
+    e = cudaFuncSetAttribute(attend_tc_kernel<D, kDecode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             TcCfg<D, kDecode>::kSmemBytes);
     if (e != cudaSuccess) return e;
-    configured = true;
+    configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
   attend_tc_kernel<D, kDecode><<<grid, kThreads, TcCfg<D, kDecode>::kSmemBytes, s>>>(km, vm, p);
