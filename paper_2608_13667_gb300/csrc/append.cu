@@ -24,7 +24,10 @@ __global__ void table_update_kernel(int32_t* __restrict__ table, const TableRun*
 // first (n_cow x L x Hkv x 16 rows x D/8, rows past the copy length idle),
 // then the appended rows in the input's own order [L][n_br][n_tok][Hkv][D/8].
 template <int D>
-__global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
+__global__ void __launch_bounds__(256) append_kernel(const AppendParams p,
+                                                     const __grid_constant__ InlineAppendPlan inl) {
+  const AppendBranch* branches = p.branches ? p.branches : inl.branches;
+  const CowCopy* cows = p.cows ? p.cows : inl.cows;
   constexpr int kChunks = D / 8;
   const int64_t cow_total = (int64_t)p.n_cow * p.L * p.Hkv * kPageTokens * kChunks;
   const int64_t app_total = (int64_t)p.L * p.n_br * p.n_tok * p.Hkv * kChunks;
@@ -37,7 +40,7 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
       const int row = (int)(x % kPageTokens); x /= kPageTokens;
       const int g = (int)(x % p.Hkv); x /= p.Hkv;
       const int l = (int)(x % p.L); x /= p.L;
-      const CowCopy cw = p.cows[x];
+      const CowCopy cw = cows[x];
       if (row >= cw.rows) continue;
       if ((uint64_t)cw.src_block >= (uint64_t)p.n_blocks ||
           (uint64_t)cw.dst_block >= (uint64_t)p.n_blocks) {
@@ -56,7 +59,7 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
       const int t = (int)(x % p.n_tok); x /= p.n_tok;
       const int b = (int)(x % p.n_br); x /= p.n_br;
       const int l = (int)x;
-      const AppendBranch br = p.branches[b];
+      const AppendBranch br = branches[b];
       const int pos = br.start + t;
       const int32_t blk = p.table[(int64_t)br.slot * p.max_pages + pos / kPageTokens];
       if ((uint64_t)blk >= (uint64_t)p.n_blocks) {
@@ -71,9 +74,13 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
 }
 
 int grid_for(int64_t total, int threads) {
+  static int sms_of[64] = {};
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (dev >= 0 && dev < 64) {
+    if (!sms_of[dev]) cudaDeviceGetAttribute(&sms_of[dev], cudaDevAttrMultiProcessorCount, dev);
+    if (sms_of[dev] > 0) sms = sms_of[dev];
+  }
   const int64_t want = (total + threads - 1) / threads;
   const int64_t cap = (int64_t)sms * 16;
   return (int)(want < 1 ? 1 : (want > cap ? cap : want));
@@ -89,15 +96,17 @@ cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int3
   return cudaGetLastError();
 }
 
-cudaError_t launch_append(const AppendParams& p, int D, cudaStream_t s) {
+cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, int D, cudaStream_t s) {
+  static const InlineAppendPlan kNone{};
+  const InlineAppendPlan& ip = inl ? *inl : kNone;
   const int64_t total = (int64_t)p.n_cow * p.L * p.Hkv * kPageTokens * (D / 8) +
                         (int64_t)p.L * p.n_br * p.n_tok * p.Hkv * (D / 8);
   if (total == 0) return cudaSuccess;
   const int grid = grid_for(total, 256);
   if (D == 128)
-    append_kernel<128><<<grid, 256, 0, s>>>(p);
+    append_kernel<128><<<grid, 256, 0, s>>>(p, ip);
   else if (D == 64)
-    append_kernel<64><<<grid, 256, 0, s>>>(p);
+    append_kernel<64><<<grid, 256, 0, s>>>(p, ip);
   else
     return cudaErrorInvalidValue;
   return cudaGetLastError();

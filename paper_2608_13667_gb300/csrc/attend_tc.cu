@@ -86,7 +86,7 @@ struct TcCfg {
 template <int D, bool kDecode>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                     const AttnParams p) {
+                     const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
   using C = TcCfg<D, kDecode>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -112,8 +112,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   // ---- what this CTA reads and for whom ------------------------------------------
   int slot, page_begin, n_pages, n_valid_keys, n_rows, min_limit, row_base = 0;
   AttnItem item{};
+  const int32_t* members = p.members ? p.members : inl.members;
   if (kDecode) {
-    item = p.items[blockIdx.x];
+    item = p.items ? p.items[blockIdx.x] : inl.items[blockIdx.x];
     slot = item.slot;
     page_begin = item.page_begin;
     n_pages = item.n_pages;
@@ -299,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   int qrow = 0, head = 0;
   if (valid) {
     if (kDecode) {
-      qrow = p.members[item.member_base + r / G];
+      qrow = members[item.member_base + r / G];
       head = kvh * G + r % G;
     } else {
       const int gr = row_base + r;
@@ -443,8 +444,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 }
 
 template <int D, bool kDecode>
-cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_ctas,
-                        cudaStream_t s) {
+cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
+                        const InlineDecodePlan& inl, int n_ctas, cudaStream_t s) {
   // the shared-memory opt-in is a per-device function attribute
   static bool configured[kMaxDevices] = {};
   int dev = 0;
@@ -458,7 +459,7 @@ cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const Attn
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  attend_tc_kernel<D, kDecode><<<grid, kThreads, TcCfg<D, kDecode>::kSmemBytes, s>>>(km, vm, p);
+  attend_tc_kernel<D, kDecode><<<grid, kThreads, TcCfg<D, kDecode>::kSmemBytes, s>>>(km, vm, p, inl);
   return cudaGetLastError();
 }
 
@@ -476,20 +477,23 @@ int decode_ctas_per_sm_t() {
 
 }  // namespace
 
-cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_items,
-                             int D, cudaStream_t s) {
+cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
+                             const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s) {
+  static const InlineDecodePlan kNone{};
+  const InlineDecodePlan& ip = inl ? *inl : kNone;
   if (n_items <= 0) return cudaSuccess;
-  if (D == 128) return launch_tc_t<128, true>(km, vm, p, n_items, s);
-  if (D == 64) return launch_tc_t<64, true>(km, vm, p, n_items, s);
+  if (D == 128) return launch_tc_t<128, true>(km, vm, p, ip, n_items, s);
+  if (D == 64) return launch_tc_t<64, true>(km, vm, p, ip, n_items, s);
   return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int D,
                             cudaStream_t s) {
+  static const InlineDecodePlan kNone{};
   if (p.T <= 0) return cudaSuccess;
   const int n_tiles = (p.T * p.G + kMmaRows - 1) / kMmaRows;
-  if (D == 128) return launch_tc_t<128, false>(km, vm, p, n_tiles, s);
-  if (D == 64) return launch_tc_t<64, false>(km, vm, p, n_tiles, s);
+  if (D == 128) return launch_tc_t<128, false>(km, vm, p, kNone, n_tiles, s);
+  if (D == 64) return launch_tc_t<64, false>(km, vm, p, kNone, n_tiles, s);
   return cudaErrorInvalidValue;
 }
 

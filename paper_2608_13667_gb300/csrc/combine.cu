@@ -16,13 +16,15 @@ namespace {
 // One warp per (layer, branch, query head): lse = log sum_i exp(lse_i),
 // O = sum_i exp(lse_i - lse) O_i over the branch's partials.
 template <int D>
-__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p) {
+__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
+                                                      const __grid_constant__ InlineDecodePlan inl) {
+  const int32_t* n_splits = p.n_splits ? p.n_splits : inl.n_splits;
   const int lane = threadIdx.x & 31;
   const int64_t idx = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
   const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
   if (idx >= total) return;
   const int b = (int)((idx / p.Hq) % p.n_br);
-  const int ns = p.n_splits[b];
+  const int ns = n_splits[b];
   const float* lse_i = p.part_lse + idx * p.max_splits;
   const float li = lane < ns ? lse_i[lane] : -INFINITY;
   float mx = li;
@@ -62,14 +64,16 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p) {
 
 }  // namespace
 
-cudaError_t launch_combine(const CombineParams& p, int D, cudaStream_t s) {
+cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, int D, cudaStream_t s) {
+  static const InlineDecodePlan kNone{};
+  const InlineDecodePlan& ip = inl ? *inl : kNone;
   const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
   if (total == 0) return cudaSuccess;
   const int grid = (int)((total + 3) / 4);
   if (D == 128)
-    combine_kernel<128><<<grid, 128, 0, s>>>(p);
+    combine_kernel<128><<<grid, 128, 0, s>>>(p, ip);
   else if (D == 64)
-    combine_kernel<64><<<grid, 128, 0, s>>>(p);
+    combine_kernel<64><<<grid, 128, 0, s>>>(p, ip);
   else
     return cudaErrorInvalidValue;
   return cudaGetLastError();

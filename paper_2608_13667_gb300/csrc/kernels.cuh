@@ -89,13 +89,31 @@ struct CombineParams {
   int32_t n_br, Hq, L, max_splits;
 };
 
+// Small per-call plans travel inside the kernel parameters (no staging copy,
+// no event): a kernel reads its plan from here when the pointer in its
+// parameter block is null.
+constexpr int kInlineItems = 64;
+constexpr int kInlineMembers = 96;
+constexpr int kInlineBranches = 64;
+struct InlineDecodePlan {
+  AttnItem items[kInlineItems];
+  int32_t members[kInlineMembers];
+  int32_t n_splits[kInlineBranches];
+};
+constexpr int kInlineAppendBranches = 32;
+constexpr int kInlineCows = 32;
+struct InlineAppendPlan {
+  AppendBranch branches[kInlineAppendBranches];
+  CowCopy cows[kInlineCows];
+};
+
 cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int32_t* values,
                                 int n_runs, cudaStream_t s);
-cudaError_t launch_append(const AppendParams& p, int D, cudaStream_t s);
-cudaError_t launch_combine(const CombineParams& p, int D, cudaStream_t s);
+cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, int D, cudaStream_t s);
+cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, int D, cudaStream_t s);
 // Decode partials on tcgen05 (one CTA per item x KV head x layer).
 cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
-                             int n_items, int D, cudaStream_t s);
+                             const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s);
 // Causal merge prefill on tcgen05 (p.slot, p.L0, p.T, p.q -> p.out_o, p.out_lse).
 cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int D,
                             cudaStream_t s);

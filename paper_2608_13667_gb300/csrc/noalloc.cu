@@ -235,7 +235,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   ap.L = c.n_layers;
   ap.max_pages = table_stride;
   ap.max_splits = kSplitStride;
-  if (launch_decode_tc(kmap, vmap, ap, n_items, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
+  if (launch_decode_tc(kmap, vmap, ap, nullptr, n_items, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
   CombineParams cp{};
   cp.part_o = ap.out_o;
   cp.part_lse = ap.out_lse;
@@ -246,6 +246,6 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   cp.Hq = c.n_q_heads;
   cp.L = c.n_layers;
   cp.max_splits = kSplitStride;
-  if (launch_combine(cp, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
+  if (launch_combine(cp, nullptr, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
   return ST_OK;
 }

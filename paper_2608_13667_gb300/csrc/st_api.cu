@@ -2,8 +2,9 @@
 //
 // The host side is authoritative: the block pool (block_pool.cpp) decides
 // every allocation, and each call turns its decision into a small plan that
-// is copied to the device through a pinned staging ring and consumed by the
-// kernels of that call.  Planning for st_decode_attn groups the branches of a
+// the kernels of that call consume -- inside their parameter block when it is
+// small (the common decode step), else copied to the device through a pinned
+// staging ring.  Planning for st_decode_attn groups the branches of a
 // call by fork family and finds the pages they share, so the kernels read a
 // shared prefix page once per group (Section 3.3 of the paper).
 #include <cudaTypedefs.h>
@@ -323,20 +324,29 @@ st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const voi
 
   st_status st = flush_tables(P, s);
   if (st != ST_OK) return st;
+  // small plans travel in the kernel parameters; larger ones through staging
+  const bool inline_plan = n_br <= kInlineAppendBranches && cows.size() <= (size_t)kInlineCows;
+  InlineAppendPlan inl;
+  const AppendBranch* d_br = nullptr;
+  const CowCopy* d_cow = nullptr;
   Plan plan;
-  int ps;
-  st = acquire_plan(P, &plan, &ps);
-  if (st != ST_OK) return st;
-  const AppendBranch* d_br;
-  AppendBranch* br = plan.alloc<AppendBranch>(n_br, &d_br);
-  const CowCopy* d_cow;
-  CowCopy* cw = plan.alloc<CowCopy>(std::max<size_t>(cows.size(), 1), &d_cow);
-  if (!br || !cw) return fail(P, ST_ERR_INVALID, "append plan does not fit the staging slot");
-  for (int i = 0; i < n_br; ++i) br[i] = AppendBranch{slots[i], starts[i]};
-  for (size_t i = 0; i < cows.size(); ++i)
-    cw[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
-  st = submit_plan(P, plan, s);
-  if (st != ST_OK) return st;
+  int ps = -1;
+  if (inline_plan) {
+    for (int i = 0; i < n_br; ++i) inl.branches[i] = AppendBranch{slots[i], starts[i]};
+    for (size_t i = 0; i < cows.size(); ++i)
+      inl.cows[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
+  } else {
+    st = acquire_plan(P, &plan, &ps);
+    if (st != ST_OK) return st;
+    AppendBranch* br = plan.alloc<AppendBranch>(n_br, &d_br);
+    CowCopy* cw = plan.alloc<CowCopy>(std::max<size_t>(cows.size(), 1), &d_cow);
+    if (!br || !cw) return fail(P, ST_ERR_INVALID, "append plan does not fit the staging slot");
+    for (int i = 0; i < n_br; ++i) br[i] = AppendBranch{slots[i], starts[i]};
+    for (size_t i = 0; i < cows.size(); ++i)
+      cw[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
+    st = submit_plan(P, plan, s);
+    if (st != ST_OK) return st;
+  }
   const st_config& c = P->cfg;
   AppendParams ap{};
   ap.k = static_cast<const __nv_bfloat16*>(k);
@@ -358,9 +368,10 @@ st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const voi
   double cow_rows = 0;
   for (auto& e : cows) cow_rows += e.rows;
   const double bytes = row_bytes * ((double)n_br * n_tok * 2 + cow_rows * 2);
-  st = run_kernel(P, kKAppend, bytes, 0, s, [&] { return launch_append(ap, c.head_dim, s); });
+  st = run_kernel(P, kKAppend, bytes, 0, s,
+                  [&] { return launch_append(ap, inline_plan ? &inl : nullptr, c.head_dim, s); });
   if (st != ST_OK) return st;
-  return retire_plan(P, ps, s);
+  return inline_plan ? ST_OK : retire_plan(P, ps, s);
 }
 
 // Longest common prefix (in pages) of two block tables.
@@ -642,11 +653,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   chunk = std::max<int64_t>(16, (chunk + 3) / 4 * 4);
   const int max_prefix_chunks = c.max_splits - 2;  // leave room for a branch's own runs
 
-  Plan plan;
-  int ps;
   st_status st = flush_tables(P, s);
-  if (st != ST_OK) return st;
-  st = acquire_plan(P, &plan, &ps);
   if (st != ST_OK) return st;
 
   std::vector<AttnItem> items;
@@ -696,18 +703,32 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   const double part_bytes = part_rows * (c.head_dim + 1) * 4;
   bytes += q_bytes + part_bytes;
 
-  const AttnItem* d_items;
-  AttnItem* hi = plan.alloc<AttnItem>(items.size(), &d_items);
-  const int32_t* d_members;
-  int32_t* hm = plan.alloc<int32_t>(members.size(), &d_members);
-  const int32_t* d_nsplit;
-  int32_t* hn = plan.alloc<int32_t>(n_br, &d_nsplit);
-  if (!hi || !hm || !hn) return fail(P, ST_ERR_INVALID, "decode plan does not fit the staging slot");
-  std::memcpy(hi, items.data(), items.size() * sizeof(AttnItem));
-  std::memcpy(hm, members.data(), members.size() * sizeof(int32_t));
-  std::memcpy(hn, n_splits.data(), n_br * sizeof(int32_t));
-  st = submit_plan(P, plan, s);
-  if (st != ST_OK) return st;
+  // small plans travel in the kernel parameters; larger ones through staging
+  const bool inline_plan = items.size() <= (size_t)kInlineItems && members.size() <= (size_t)kInlineMembers &&
+                           n_br <= kInlineBranches;
+  InlineDecodePlan inl;
+  const AttnItem* d_items = nullptr;
+  const int32_t* d_members = nullptr;
+  const int32_t* d_nsplit = nullptr;
+  Plan plan;
+  int ps = -1;
+  if (inline_plan) {
+    std::memcpy(inl.items, items.data(), items.size() * sizeof(AttnItem));
+    std::memcpy(inl.members, members.data(), members.size() * sizeof(int32_t));
+    std::memcpy(inl.n_splits, n_splits.data(), n_br * sizeof(int32_t));
+  } else {
+    st = acquire_plan(P, &plan, &ps);
+    if (st != ST_OK) return st;
+    AttnItem* hi = plan.alloc<AttnItem>(items.size(), &d_items);
+    int32_t* hm = plan.alloc<int32_t>(members.size(), &d_members);
+    int32_t* hn = plan.alloc<int32_t>(n_br, &d_nsplit);
+    if (!hi || !hm || !hn) return fail(P, ST_ERR_INVALID, "decode plan does not fit the staging slot");
+    std::memcpy(hi, items.data(), items.size() * sizeof(AttnItem));
+    std::memcpy(hm, members.data(), members.size() * sizeof(int32_t));
+    std::memcpy(hn, n_splits.data(), n_br * sizeof(int32_t));
+    st = submit_plan(P, plan, s);
+    if (st != ST_OK) return st;
+  }
 
   AttnParams ap{};
   ap.q = static_cast<const __nv_bfloat16*>(q);
@@ -729,7 +750,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
   const int n_items = (int)items.size();
   st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
-    return launch_decode_tc(P->kmap, P->vmap, ap, n_items, c.head_dim, s);
+    return launch_decode_tc(P->kmap, P->vmap, ap, inline_plan ? &inl : nullptr, n_items, c.head_dim, s);
   });
   if (st != ST_OK) return st;
 
@@ -744,9 +765,10 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   cp.L = c.n_layers;
   cp.max_splits = c.max_splits;
   const double cbytes = part_bytes + (double)c.n_layers * n_br * c.n_q_heads * (c.head_dim + 1) * 4;
-  st = run_kernel(P, kKCombine, cbytes, 0, s, [&] { return launch_combine(cp, c.head_dim, s); });
+  st = run_kernel(P, kKCombine, cbytes, 0, s,
+                  [&] { return launch_combine(cp, inline_plan ? &inl : nullptr, c.head_dim, s); });
   if (st != ST_OK) return st;
-  return retire_plan(P, ps, s);
+  return inline_plan ? ST_OK : retire_plan(P, ps, s);
 }
 
 ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, const void* k,
