@@ -36,23 +36,41 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
   for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
   const float lse = mx + logf(sum);
   constexpr int kPer = D / 32;
+  constexpr int kBatch = 8;  // partials whose loads are in flight together
+  const float inv_sum = 1.f / sum;
   float out[kPer];
 #pragma unroll
   for (int e = 0; e < kPer; ++e) out[e] = 0.f;
   const float* po = p.part_o + idx * p.max_splits * D + lane * kPer;
-  for (int i = 0; i < ns; ++i) {
-    const float wi = __shfl_sync(0xffffffffu, w, i) / sum;
-    if (kPer == 4) {
-      const float4 x = *reinterpret_cast<const float4*>(po + (int64_t)i * D);
-      out[0] += wi * x.x;
-      out[1] += wi * x.y;
-      out[2] += wi * x.z;
-      out[3] += wi * x.w;
-    } else {
-      const float2 x = *reinterpret_cast<const float2*>(po + (int64_t)i * D);
-      out[0] += wi * x.x;
-      out[1] += wi * x.y;
+  for (int i0 = 0; i0 < ns; i0 += kBatch) {
+    float x[kBatch][kPer];
+    float wv[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int i = i0 + u;
+      wv[u] = __shfl_sync(0xffffffffu, w, i & 31) * inv_sum;
+      if (i < ns) {
+        if constexpr (kPer == 4) {
+          const float4 v = *reinterpret_cast<const float4*>(po + (int64_t)i * D);
+          x[u][0] = v.x;
+          x[u][1] = v.y;
+          x[u][2] = v.z;
+          x[u][3] = v.w;
+        } else {
+          const float2 v = *reinterpret_cast<const float2*>(po + (int64_t)i * D);
+          x[u][0] = v.x;
+          x[u][1] = v.y;
+        }
+      } else {
+        wv[u] = 0.f;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) x[u][e] = 0.f;
+      }
     }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u)
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) out[e] += wv[u] * x[u][e];
   }
   float* dst = p.o + idx * D + lane * kPer;
   if (kPer == 4)
