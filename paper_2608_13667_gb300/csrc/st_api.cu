@@ -651,7 +651,8 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   const int64_t target_ctas = (int64_t)32 * P->sms * P->decode_ctas_per_sm;
   int64_t chunk = (units + target_ctas - 1) / target_ctas;
   chunk = std::max<int64_t>(16, (chunk + 3) / 4 * 4);
-  const int max_prefix_chunks = c.max_splits - 2;  // leave room for a branch's own runs
+  // leave room for a branch's own runs, but never fewer than one run for the prefix
+  const int max_prefix_chunks = std::max(1, c.max_splits - 2);
 
   st_status st = flush_tables(P, s);
   if (st != ST_OK) return st;

@@ -73,7 +73,7 @@ class Run:
         k, v = kv_rows(w, tag, n * n_tok, device=self.device)
         shape = (w.n_layers, n, n_tok, w.n_kv_heads, w.head_dim)
         self.pool.append_kv([self.handle[r] for r in rids], k.view(shape), v.view(shape))
-        self.ref.append(rids, n_tok)
+        self.ref.append(rids, n_tok)  # the library accepted it, so the reference must too
         self.sizes[tag] = n * n_tok
         for i, r in enumerate(rids):
             self.hist[r].append((tag, i * n_tok, n_tok))
