@@ -35,7 +35,8 @@
 // Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
 //   Q  [D/64][rows][64]       K-major A (SBO 1024)
 //   K  [D/64][keys][64]       K-major B (SBO 1024)
-//   P  [rows][keys]           K-major A (SBO 1024), written over K
+//   P  [rows][keys]           K-major A (SBO 1024), written over K (decode:
+//                             two bf16 terms P_hi, P_lo, one after the other)
 //   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
 // The MMA always computes 128 rows.  In decode only the first <= 48 Q and P
 // rows are written; rows past them read whatever follows in shared memory and
@@ -63,7 +64,7 @@ constexpr int kMaxDevices = 64;
 
 constexpr int cmax(int a, int b) { return a > b ? a : b; }
 
-template <int D, bool kDecode>
+template <int D, bool kDecode, bool kSplit = kDecode>
 struct TcCfg {
   static constexpr int kHalves = D / 64;
   static constexpr int kKeys = 64;                     // keys per stage
@@ -73,21 +74,29 @@ struct TcCfg {
   static constexpr int kQHalfBytes = kQRows * 128;
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kKVHalfBytes = kKeys * 128;
-  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, kQRows * 128);  // K, then P
+  // P as two bf16 terms (P = P_hi + P_lo, two MMAs against the same V): with
+  // few keys the rounding of a single bf16 P does not average out.  Decode
+  // always splits; the merge splits only when its rows see few keys (the
+  // second term costs it a second CTA per SM).
+  static constexpr bool kSplitP = kSplit;
+  static constexpr int kPTermBytes = kQRows * 128;                // one term, kQRows rows
+  static constexpr int kPloOffset = kSplitP ? kPTermBytes : 0;    // P_lo after P_hi in the K slot
+  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, (kSplitP ? 2 : 1) * kPTermBytes);
   static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
   static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
-  // the MMA reads 128 rows of P from the last K slot: keep that inside the allocation
-  static constexpr int kOverread = cmax(0, kMmaRows * 128 - kStageBytes);
+  // the MMA reads 128 rows of each P term from the last K slot: keep that
+  // inside the allocation
+  static constexpr int kOverread = cmax(0, kPloOffset + kMmaRows * 128 - kStageBytes);
   static constexpr int kBarOffset = kQBytes + kRingBytes + kOverread;
   static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 };
 
-template <int D, bool kDecode>
+template <int D, bool kDecode, bool kSplit>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
-  using C = TcCfg<D, kDecode>;
+  using C = TcCfg<D, kDecode, kSplit>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
@@ -275,6 +284,12 @@ __global__ void __launch_bounds__(kThreads, 2)
           tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + ks * 32, 16, 1024),
                       tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
                       (j > 0 || ks > 0) ? 1u : 0u);
+        if constexpr (C::kSplitP) {
+#pragma unroll
+          for (int ks = 0; ks < C::kKeys / 16; ++ks)
+            tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
+                        tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
+        }
         tc_commit(&empty[s]);
         tc_commit(o_ready);
         if (jn < n_tiles && !early && !issue_s(jn)) {
@@ -378,18 +393,26 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint8_t* kslot = ring + s * C::kStageBytes;  // S_j has been consumed: P_j goes over K_j
     if (valid) {
       uint32_t pk[C::kKeys / 2];
+      uint32_t pl[C::kSplitP ? C::kKeys / 2 : 1];
       float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < C::kKeys; c += 2) {
         const float a = ex2(fmaf(sc[c], sl2, -m_used)), b = ex2(fmaf(sc[c + 1], sl2, -m_used));
         rs[(c >> 1) & 7] += a + b;
-        pk[c / 2] = pack_bf16(a, b);
+        const uint32_t hi = pack_bf16(a, b);
+        pk[c / 2] = hi;
+        if constexpr (C::kSplitP)  // remainders below the bf16 rounding of a and b
+          pl[c / 2] = pack_bf16(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
       }
       l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
 #pragma unroll
-      for (int c = 0; c < C::kKeys / 8; ++c)
-        *reinterpret_cast<uint4*>(kslot + r * 128 + ((c ^ (r & 7)) << 4)) =
-            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+      for (int c = 0; c < C::kKeys / 8; ++c) {
+        const uint32_t off = r * 128 + ((c ^ (r & 7)) << 4);
+        *reinterpret_cast<uint4*>(kslot + off) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        if constexpr (C::kSplitP)
+          *reinterpret_cast<uint4*>(kslot + C::kPloOffset + off) =
+              make_uint4(pl[4 * c], pl[4 * c + 1], pl[4 * c + 2], pl[4 * c + 3]);
+      }
     }
     if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
       // this stage's copies have landed (S_j was computed from them): zero
@@ -443,9 +466,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   named_barrier_sync(1, n_swt + 32);
 }
 
-template <int D, bool kDecode>
+template <int D, bool kDecode, bool kSplit>
 cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
                         const InlineDecodePlan& inl, int n_ctas, cudaStream_t s) {
+  using C = TcCfg<D, kDecode, kSplit>;
   // the shared-memory opt-in is a per-device function attribute
   static bool configured[kMaxDevices] = {};
   int dev = 0;
@@ -453,27 +477,31 @@ cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const Attn
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    e = cudaFuncSetAttribute(attend_tc_kernel<D, kDecode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             TcCfg<D, kDecode>::kSmemBytes);
+    e = cudaFuncSetAttribute(attend_tc_kernel<D, kDecode, kSplit>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  attend_tc_kernel<D, kDecode><<<grid, kThreads, TcCfg<D, kDecode>::kSmemBytes, s>>>(km, vm, p, inl);
+  attend_tc_kernel<D, kDecode, kSplit><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
   return cudaGetLastError();
 }
 
 template <int D>
 int decode_ctas_per_sm_t() {
-  if (cudaFuncSetAttribute(attend_tc_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           TcCfg<D, true>::kSmemBytes) != cudaSuccess)
+  using C = TcCfg<D, true>;
+  if (cudaFuncSetAttribute(attend_tc_kernel<D, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           C::kSmemBytes) != cudaSuccess)
     return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, true>, kThreads,
-                                                    TcCfg<D, true>::kSmemBytes) != cudaSuccess)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, true, true>, kThreads,
+                                                    C::kSmemBytes) != cudaSuccess)
     return 0;
   return n < 2 ? n : 2;  // two CTAs' TMEM (2 x 256 columns) fill an SM
 }
+
+// Merges whose longest row sees at most this many keys use two P terms.
+constexpr int kMergeSplitMaxKeys = 2048;
 
 }  // namespace
 
@@ -482,8 +510,8 @@ cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const
   static const InlineDecodePlan kNone{};
   const InlineDecodePlan& ip = inl ? *inl : kNone;
   if (n_items <= 0) return cudaSuccess;
-  if (D == 128) return launch_tc_t<128, true>(km, vm, p, ip, n_items, s);
-  if (D == 64) return launch_tc_t<64, true>(km, vm, p, ip, n_items, s);
+  if (D == 128) return launch_tc_t<128, true, true>(km, vm, p, ip, n_items, s);
+  if (D == 64) return launch_tc_t<64, true, true>(km, vm, p, ip, n_items, s);
   return cudaErrorInvalidValue;
 }
 
@@ -492,8 +520,13 @@ cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const 
   static const InlineDecodePlan kNone{};
   if (p.T <= 0) return cudaSuccess;
   const int n_tiles = (p.T * p.G + kMmaRows - 1) / kMmaRows;
-  if (D == 128) return launch_tc_t<128, false>(km, vm, p, kNone, n_tiles, s);
-  if (D == 64) return launch_tc_t<64, false>(km, vm, p, kNone, n_tiles, s);
+  const bool split = (int64_t)p.L0 + p.T <= kMergeSplitMaxKeys;
+  if (D == 128)
+    return split ? launch_tc_t<128, false, true>(km, vm, p, kNone, n_tiles, s)
+                 : launch_tc_t<128, false, false>(km, vm, p, kNone, n_tiles, s);
+  if (D == 64)
+    return split ? launch_tc_t<64, false, true>(km, vm, p, kNone, n_tiles, s)
+                 : launch_tc_t<64, false, false>(km, vm, p, kNone, n_tiles, s);
   return cudaErrorInvalidValue;
 }
 
