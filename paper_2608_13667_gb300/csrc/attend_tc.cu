@@ -70,6 +70,11 @@ struct TcCfg {
   static constexpr int kKeys = 64;                     // keys per stage
   static constexpr int kPagesPerStage = kKeys / kPageTokens;
   static constexpr int kStages = kDecode ? 3 : 2;
+  // MMA M: decode stacks <= 48 rows and uses M = 64, whose accumulator rows
+  // sit in TMEM lanes 0..15 of each warp's 32-lane quarter (row r at lane
+  // 32 * (r / 16) + r % 16); the merge uses M = 128 (row r at lane r).
+  static constexpr int kM = kDecode ? 64 : 128;
+  static constexpr int kRowsPerWarp = kM / 4;
   static constexpr int kQRows = kDecode ? 48 : 128;    // Q/P rows stored
   static constexpr int kQHalfBytes = kQRows * 128;
   static constexpr int kQBytes = kHalves * kQHalfBytes;
@@ -85,9 +90,9 @@ struct TcCfg {
   static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
   static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
-  // the MMA reads 128 rows of each P term from the last K slot: keep that
+  // the MMA reads kM rows of each P term from the last K slot: keep that
   // inside the allocation
-  static constexpr int kOverread = cmax(0, kPloOffset + kMmaRows * 128 - kStageBytes);
+  static constexpr int kOverread = cmax(0, kPloOffset + kM * 128 - kStageBytes);
   static constexpr int kBarOffset = kQBytes + kRingBytes + kOverread;
   static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 };
@@ -142,7 +147,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     min_limit = p.L0 + t_first + 1;
   }
   const int n_tiles = (n_pages + C::kPagesPerStage - 1) / C::kPagesPerStage;
-  const int n_sw = (n_rows + 31) >> 5;   // softmax warps with rows
+  const int n_sw = (n_rows + C::kRowsPerWarp - 1) / C::kRowsPerWarp;  // softmax warps with rows
   const int n_swt = n_sw * 32;
 
   if (threadIdx.x == 0) {
@@ -234,8 +239,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   // ---- MMA issuer ----------------------------------------------------------------
   if (warp == kMmaWarp) {
     if (lane == 0) {
-      constexpr uint32_t idesc_s = tc_idesc_bf16(kMmaRows, C::kKeys, 0, 0);
-      constexpr uint32_t idesc_o = tc_idesc_bf16(kMmaRows, D, 0, 1);
+      constexpr uint32_t idesc_s = tc_idesc_bf16(C::kM, C::kKeys, 0, 0);
+      constexpr uint32_t idesc_o = tc_idesc_bf16(C::kM, D, 0, 1);
       const uint32_t q_addr = smem_addr(q_s);
       bool ok = mbar_wait(q_ready, 0);
       tc_fence_after_sync();
@@ -309,7 +314,17 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (warp >= n_sw) return;
 
   // ---- softmax warps ---------------------------------------------------------------
-  const int r = threadIdx.x;
+  // Merge (M = 128): thread r owns row r (TMEM lane r), all of its keys and O
+  // columns.  Decode (M = 64): the rows sit in lanes 0..15 of each warp's
+  // quarter and threads t and t + 16 share row t: half of the stage's keys
+  // and half of the O columns each (16-lane TMEM loads with a column split),
+  // the row max and sum combined with one shuffle.
+  constexpr bool kPair = C::kM == 64;
+  constexpr int kKpt = C::kKeys / (kPair ? 2 : 1);  // keys per thread per stage
+  constexpr int kOpt = D / (kPair ? 2 : 1);         // O columns per thread
+  const int tid = threadIdx.x;                      // 0 .. n_swt-1, for cooperative loops
+  const int half = kPair ? (lane >> 4) : 0;
+  const int r = kPair ? warp * 16 + (lane & 15) : threadIdx.x;  // this thread's row
   const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
   const bool valid = r < n_rows;
   int qrow = 0, head = 0;
@@ -326,8 +341,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int limit = (!kDecode && valid) ? p.L0 + qrow + 1 : n_valid_keys;
   if (r < C::kQRows) {
     const uint4* src = reinterpret_cast<const uint4*>(p.q + (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * D);
+    constexpr int kChunks = D / 8 / (kPair ? 2 : 1);  // 16-byte chunks of the row this thread writes
 #pragma unroll
-    for (int c = 0; c < D / 8; ++c) {
+    for (int cc = 0; cc < kChunks; ++cc) {
+      const int c = half * kChunks + cc;
       const uint4 v = valid ? src[c] : make_uint4(0u, 0u, 0u, 0u);
       *reinterpret_cast<uint4*>(q_s + (c >> 3) * C::kQHalfBytes + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
     }
@@ -335,8 +352,19 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   mbar_arrive(q_ready);
 
+  // this thread's 32-column pieces of its O row: [o_col(k), o_col(k) + 32)
+  auto o_load = [&](int k, float* o) {
+    if constexpr (kPair) tmem_ld16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
+    else tmem_ld32(t_lane + kTmemO + k * 32, o);
+  };
+  auto o_store = [&](int k, const float* o) {
+    if constexpr (kPair) tmem_st16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
+    else tmem_st32(t_lane + kTmemO + k * 32, o);
+  };
+  auto o_col = [&](int k) { return half * (D / 2) + k * 32; };
+
   const float sl2 = p.scale_log2;
-  float m_used = -1e30f, l = 0.f;
+  float m_used = -1e30f, l = 0.f;  // l: this thread's share of the row sum
   bool ok = true;
   for (int j = 0; j < n_tiles; ++j) {
     const int s = j % C::kStages;
@@ -345,27 +373,31 @@ __global__ void __launch_bounds__(kThreads, 2)
       break;
     }
     tc_fence_after_sync();
-    // raw scores q.k; the softmax works in the log2 domain, x = s * sl2
-    float sc[C::kKeys];
-    static_assert(C::kKeys == 64, "one 64-column TMEM load per stage");
-    tmem_ld64(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
+    // raw scores q.k of this thread's keys; the softmax works in the log2
+    // domain, x = s * sl2
+    float sc[kKpt];
+    static_assert(C::kKeys == 64, "64 keys per stage");
+    if constexpr (kPair) tmem_ld16x2_32<32>(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
+    else tmem_ld64(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
     const int key0 = j * C::kKeys;
+    const int kbase = half * kKpt;  // this thread's first key within the stage
     const int np = min(C::kPagesPerStage, n_pages - j * C::kPagesPerStage);
     const int loaded = np * kPageTokens;
     const bool edge = key0 + C::kKeys > min_limit || loaded < C::kKeys;
     if (edge) {
 #pragma unroll
-      for (int c = 0; c < C::kKeys; ++c)
-        if (c >= loaded || key0 + c >= limit) sc[c] = -INFINITY;
+      for (int c = 0; c < kKpt; ++c)
+        if (kbase + c >= loaded || key0 + kbase + c >= limit) sc[c] = -INFINITY;
     }
     // 8 independent max chains, then a tree (short dependency chains)
     float mx8[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) mx8[i] = sc[i];
 #pragma unroll
-    for (int c = 8; c < C::kKeys; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sc[c]);
-    const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                           fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+    for (int c = 8; c < kKpt; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sc[c]);
+    float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                     fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+    if constexpr (kPair) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
     const float m_new = fmaxf(m_used, mx * sl2);  // sl2 > 0: max commutes with the scale
     const bool need = valid && m_new > m_used + kRescaleThreshold;
     if (__any_sync(0xffffffffu, need)) {
@@ -379,12 +411,12 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         tc_fence_after_sync();
 #pragma unroll 1
-        for (int c0 = 0; c0 < D; c0 += 32) {
+        for (int k = 0; k < kOpt / 32; ++k) {
           float o[32];
-          tmem_ld32(t_lane + kTmemO + c0, o);
+          o_load(k, o);
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st32(t_lane + kTmemO + c0, o);
+          o_store(k, o);
         }
       }
       l *= alpha;
@@ -392,11 +424,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     uint8_t* kslot = ring + s * C::kStageBytes;  // S_j has been consumed: P_j goes over K_j
     if (valid) {
-      uint32_t pk[C::kKeys / 2];
-      uint32_t pl[C::kSplitP ? C::kKeys / 2 : 1];
+      uint32_t pk[kKpt / 2];
+      uint32_t pl[C::kSplitP ? kKpt / 2 : 1];
       float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < C::kKeys; c += 2) {
+      for (int c = 0; c < kKpt; c += 2) {
         const float a = ex2(fmaf(sc[c], sl2, -m_used)), b = ex2(fmaf(sc[c + 1], sl2, -m_used));
         rs[(c >> 1) & 7] += a + b;
         const uint32_t hi = pack_bf16(a, b);
@@ -406,12 +438,13 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
 #pragma unroll
-      for (int c = 0; c < C::kKeys / 8; ++c) {
+      for (int cc = 0; cc < kKpt / 8; ++cc) {
+        const int c = half * (kKpt / 8) + cc;  // 16-byte chunk of the P row (8 keys)
         const uint32_t off = r * 128 + ((c ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4*>(kslot + off) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        *reinterpret_cast<uint4*>(kslot + off) = make_uint4(pk[4 * cc], pk[4 * cc + 1], pk[4 * cc + 2], pk[4 * cc + 3]);
         if constexpr (C::kSplitP)
           *reinterpret_cast<uint4*>(kslot + C::kPloOffset + off) =
-              make_uint4(pl[4 * c], pl[4 * c + 1], pl[4 * c + 2], pl[4 * c + 3]);
+              make_uint4(pl[4 * cc], pl[4 * cc + 1], pl[4 * cc + 2], pl[4 * cc + 3]);
       }
     }
     if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
@@ -419,7 +452,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       // the V rows of keys that are not valid
       mbar_wait(&full[s], (j / C::kStages) & 1);
       uint8_t* vslot = kslot + C::kKSlotBytes;
-      for (int t = r; t < C::kKeys * C::kHalves; t += n_swt) {
+      for (int t = tid; t < C::kKeys * C::kHalves; t += n_swt) {
         const int c = t % C::kKeys, h = t / C::kKeys;
         if (c >= loaded || key0 + c >= n_valid_keys) {
 #pragma unroll
@@ -435,6 +468,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0));
   tc_fence_after_sync();
   if (ok) {
+    if constexpr (kPair) l += __shfl_xor_sync(0xffffffffu, l, 16);  // the row's full sum
     const float inv = 1.f / l;
     float* dst = nullptr;
     float* dst_lse = nullptr;
@@ -445,16 +479,16 @@ __global__ void __launch_bounds__(kThreads, 2)
       else
         idx = ((int64_t)layer * p.T + qrow) * p.Hq + head;
       dst = p.out_o + idx * D;
-      dst_lse = p.out_lse + idx;
+      if (half == 0) dst_lse = p.out_lse + idx;
     }
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 32) {
+    for (int k = 0; k < kOpt / 32; ++k) {
       float o[32];
-      tmem_ld32(t_lane + kTmemO + c0, o);
+      o_load(k, o);
       if (dst) {
 #pragma unroll
         for (int i = 0; i < 32; i += 4)
-          *reinterpret_cast<float4*>(dst + c0 + i) =
+          *reinterpret_cast<float4*>(dst + o_col(k) + i) =
               make_float4(o[i] * inv, o[i + 1] * inv, o[i + 2] * inv, o[i + 3] * inv);
       }
     }
