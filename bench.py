@@ -316,6 +316,24 @@ def run_profile_small():
         pool.decode_attn(br, queries(w, ("q", s), n, device=dev), o, lse)
     pool.sync()
     d = pool.profile_read()["decode_partial"]
+    pool.close()
+    del pool
+    mg = _merge_case()
+    print(json.dumps({"decode_ms_per_launch": d["total_ms"] / d["launches"],
+                      "decode_gbs": d["bytes"] / d["total_ms"] / 1e6, **mg}))
+
+
+def _merge_case(n_merges=3):
+    """Merges of 2048 thought rows onto a 16896-token main context (32 q / 8 kv
+    heads, D 128, 4 layers): main is forked n_merges times and each fork takes
+    one merge, so every launch does the same work.  Returns the CUDA-event
+    timing of the fastest launch."""
+    import dataclasses
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import get, kv_rows, queries
+    dev = torch.device("cuda", 0)
+    st.build()
     w5 = dataclasses.replace(get(5), n_layers=4)
     p5 = st.Pool(n_layers=4, n_q_heads=w5.n_q_heads, n_kv_heads=w5.n_kv_heads, head_dim=w5.head_dim,
                  n_blocks=4096, seed=1, device=dev, max_seqs=8, max_pages=2048, max_decode_branches=8,
@@ -324,15 +342,27 @@ def run_profile_small():
     for c0 in range(0, 16896, 8448):
         k, v = kv_rows(w5, ("ctx", c0), 8448, device=dev)
         p5.append_kv([m], k.view(4, 1, 8448, 8, 128), v.view(4, 1, 8448, 8, 128))
+    forks = p5.fork(m, n_merges)
     k, v = kv_rows(w5, ("merge",), 2048, device=dev)
     q = queries(w5, ("mq",), 2048, device=dev)
-    p5.profile_enable(True)
-    p5.merge(m, q, k, v)
-    p5.sync()
-    mg = p5.profile_read()["merge_prefill"]
-    print(json.dumps({"decode_ms_per_launch": d["total_ms"] / d["launches"],
-                      "decode_gbs": d["bytes"] / d["total_ms"] / 1e6,
-                      "merge_ms": mg["total_ms"], "merge_tflops": mg["flops"] / mg["total_ms"] / 1e9}))
+    best = None
+    for f in forks:
+        p5.profile_enable(True)
+        p5.merge(f, q, k, v)
+        p5.sync()
+        mg = p5.profile_read()["merge_prefill"]
+        p5.profile_enable(False)
+        if best is None or mg["total_ms"] < best["total_ms"]:
+            best = mg
+    p5.close()
+    return {"merge_ms": best["total_ms"], "merge_tflops": best["flops"] / best["total_ms"] / 1e9,
+            "merges": n_merges}
+
+
+def run_profile_merge():
+    """Only the merge case of run_profile_small (about 1 GB on the device):
+    three identical merge launches, for ncu captures of the merge kernel."""
+    print(json.dumps(_merge_case()))
 
 
 def run_cycle():
@@ -479,11 +509,16 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-small", action="store_true",
                     help="run the small decode + merge case used for ncu captures and exit")
+    ap.add_argument("--profile-merge", action="store_true",
+                    help="run only the merge case of --profile-small (three identical launches) and exit")
     ap.add_argument("--cycle", action="store_true",
                     help="time the full fork/decode/merge cycle workload and exit")
     args = ap.parse_args()
     if args.profile_small:
         run_profile_small()
+        return
+    if args.profile_merge:
+        run_profile_merge()
         return
     if args.cycle:
         run_cycle()

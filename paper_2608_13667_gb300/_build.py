@@ -18,7 +18,7 @@ LIB = os.path.join(HERE, "libsecondthought.so")
 OBJDIR = os.path.join(HERE, "_build")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["block_pool.cpp", "append.cu", "attend_tc.cu", "combine.cu", "st_api.cu", "noalloc.cu", "harvest.cu"]
+SOURCES = ["block_pool.cpp", "append.cu", "attend_tc.cu", "merge_tc.cu", "combine.cu", "st_api.cu", "noalloc.cu", "harvest.cu"]
 
 
 def _nvcc():

@@ -553,14 +553,11 @@ cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const 
                             cudaStream_t s) {
   static const InlineDecodePlan kNone{};
   if (p.T <= 0) return cudaSuccess;
+  // long contexts: two query tiles per CTA sharing K/V (merge_tc.cu)
+  if ((int64_t)p.L0 + p.T > kMergeSplitMaxKeys) return launch_merge_pair(km, vm, p, D, s);
   const int n_tiles = (p.T * p.G + kMmaRows - 1) / kMmaRows;
-  const bool split = (int64_t)p.L0 + p.T <= kMergeSplitMaxKeys;
-  if (D == 128)
-    return split ? launch_tc_t<128, false, true>(km, vm, p, kNone, n_tiles, s)
-                 : launch_tc_t<128, false, false>(km, vm, p, kNone, n_tiles, s);
-  if (D == 64)
-    return split ? launch_tc_t<64, false, true>(km, vm, p, kNone, n_tiles, s)
-                 : launch_tc_t<64, false, false>(km, vm, p, kNone, n_tiles, s);
+  if (D == 128) return launch_tc_t<128, false, true>(km, vm, p, kNone, n_tiles, s);
+  if (D == 64) return launch_tc_t<64, false, true>(km, vm, p, kNone, n_tiles, s);
   return cudaErrorInvalidValue;
 }
 
