@@ -36,11 +36,12 @@
 // Synchronisation (every wait bounded; a wait that runs out sets the status
 // word and the CTA winds down):
 //   k_full / k_empty, v_full / v_empty   ring slots (TMA bytes / MMA commit)
-//   s_full[t]   S_t of the stage is complete                    (MMA commit)
-//   p_full[t]   P_t of the stage is in TMEM                     (128 arrivals)
-//   o_final     every MMA of the CTA has completed
-// S_t(j + 1) is issued only after p_full[t] of stage j, so each barrier is
-// at most one phase ahead of its waiters.
+//   s_full[t]      S_t of the stage is complete                 (MMA commit)
+//   p_full[t][h]   P_t of keys [64 h, 64 h + 64) is in TMEM     (128 arrivals)
+//   o_final        every MMA of the CTA has completed
+// S_t(j + 1) is issued only after p_full[t][1] of stage j, so each barrier is
+// at most one phase ahead of its waiters.  The MMAs of the first half of P
+// run while the softmax computes the second.
 //
 // Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
 //   Q_t [D/64][128 rows][64]   K-major A (SBO 1024)
@@ -50,6 +51,8 @@
 // last stage did not load) are zeroed by tile A's threads before P V, so that
 // stale shared or pool memory cannot turn 0 * x into NaN in a real row.
 #include <math.h>
+
+#include <type_traits>
 
 #include "kernels.cuh"
 #include "ptx.cuh"
@@ -107,8 +110,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* v_full = k_empty + kKS;
   uint64_t* v_empty = v_full + kVS;
   uint64_t* s_full = v_empty + kVS;  // [2 tiles]
-  uint64_t* p_full = s_full + 2;     // [2 tiles]
-  uint64_t* o_final = p_full + 2;
+  uint64_t* p_full = s_full + 2;     // [2 tiles][2 key halves]
+  uint64_t* o_final = p_full + 4;
   uint64_t* q_ready = o_final + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_ready + 1);
 
@@ -136,7 +139,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(&s_full[t], 1);
-      mbar_init(&p_full[t], kTileRows);
+      mbar_init(&p_full[2 * t], kTileRows);
+      mbar_init(&p_full[2 * t + 1], kTileRows);
     }
     mbar_init(o_final, 1);
     mbar_init(q_ready, kSoftThreads);
@@ -212,57 +216,78 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ---- MMA issuer ----------------------------------------------------------------
+  // One thread issues every MMA (two issuers interleaving on the tensor pipe
+  // measured slower).  It shares its sub-partition with two softmax warps, so
+  // the per-MMA work is kept to a constant add: a shared-memory descriptor's
+  // start field holds address / 16 (below 2^14 here), so the descriptor of an
+  // operand shifted by b bytes is the base descriptor + b / 16.
   if (warp == kMmaWarp) {
     if (lane == 0) {
       constexpr uint32_t idesc_s = tc_idesc_bf16(kTileRows, kKeys, 0, 0);
       constexpr uint32_t idesc_o = tc_idesc_bf16(kTileRows, D, 0, 1);
-      const uint32_t q_addr = smem_addr(base + C::kQOff);
+      const uint64_t q_desc = tc_desc_sw128(smem_addr(base + C::kQOff), 16, 1024);
+      const uint64_t k_desc0 = tc_desc_sw128(smem_addr(base + C::kKOff), 16, 1024);
+      const uint64_t v_desc0 = tc_desc_sw128(smem_addr(base + C::kVOff), C::kKVHalfBytes, 1024);
       bool ok = mbar_wait(q_ready, 0);
       tc_fence_after_sync();
-      // O_t += P_t(i) V_i, P_t(i) read from TMEM over S_t(i)
-      auto issue_pv = [&](int t, int i) -> bool {
+      // O_t += P_t(i) V_i, P_t(i) read from TMEM over S_t(i); each half of P
+      // (64 keys) is published on its own, so the first half's MMAs run while
+      // the softmax finishes the second
+      auto issue_pv = [&](auto tile, int i) -> bool {
+        constexpr int t = decltype(tile)::value;
         const int s = i % kVS;
         if (t == 0 && !mbar_wait(&v_full[s], (i / kVS) & 1)) return false;
-        if (!mbar_wait(&p_full[t], i & 1)) return false;
-        tc_fence_after_sync();
-        const uint32_t v_addr = smem_addr(base + C::kVOff + s * C::kSlotBytes);
+        const uint64_t vd = v_desc0 + (uint64_t)((s * C::kSlotBytes) >> 4);
+        const uint32_t acc0 = i > 0 ? 1u : 0u;
 #pragma unroll
-        for (int ks = 0; ks < kKeys / 16; ++ks)
-          tc_mma_bf16_tmem_a(tmem + t * kTmemTile + kTmemO, tmem + t * kTmemTile + ks * 8,
-                             tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
-                             (i > 0 || ks > 0) ? 1u : 0u);
+        for (int hf = 0; hf < 2; ++hf) {
+          if (!mbar_wait(&p_full[2 * t + hf], i & 1)) return false;
+          tc_fence_after_sync();
+#pragma unroll
+          for (int kq = 0; kq < kKeys / 32; ++kq) {
+            const int ks = hf * (kKeys / 32) + kq;
+            tc_mma_bf16_tmem_a(tmem + t * kTmemTile + kTmemO, tmem + t * kTmemTile + ks * 8,
+                               vd + (uint64_t)((ks * 16 * 128) >> 4), idesc_o, ks > 0 ? 1u : acc0);
+          }
+        }
         if (t == 1) tc_commit(&v_empty[s]);
         return true;
       };
+      // S_t(j) = Q_t K_j^T
+      auto issue_s = [&](auto tile, uint64_t kd) {
+        constexpr int t = decltype(tile)::value;
+#pragma unroll
+        for (int h = 0; h < C::kHalves; ++h)
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16(tmem + t * kTmemTile,
+                        q_desc + (uint64_t)((t * C::kQTileBytes + h * C::kQHalfBytes + kk * 32) >> 4),
+                        kd + (uint64_t)((h * C::kKVHalfBytes + kk * 32) >> 4), idesc_s, (h | kk) != 0);
+        tc_commit(&s_full[t]);
+      };
+      const std::integral_constant<int, 0> tile_a;
+      const std::integral_constant<int, 1> tile_b;
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int s = j % kKS;
-        const uint32_t k_addr = smem_addr(base + C::kKOff + s * C::kSlotBytes);
-        for (int t = 0; t < 2 && ok; ++t) {
-          if (j > 0 && !issue_pv(t, j - 1)) {
-            ok = false;
-            break;
-          }
-          if (t == 0) {
-            if (!mbar_wait(&k_full[s], (j / kKS) & 1)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after_sync();
-          }
-#pragma unroll
-          for (int h = 0; h < C::kHalves; ++h)
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc_mma_bf16(tmem + t * kTmemTile,
-                          tc_desc_sw128(q_addr + t * C::kQTileBytes + h * C::kQHalfBytes + kk * 32, 16, 1024),
-                          tc_desc_sw128(k_addr + h * C::kKVHalfBytes + kk * 32, 16, 1024), idesc_s,
-                          (h | kk) != 0);
-          tc_commit(&s_full[t]);
+        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kSlotBytes) >> 4);
+        if (j > 0 && !issue_pv(tile_a, j - 1)) {
+          ok = false;
+          break;
         }
-        if (ok) tc_commit(&k_empty[s]);
+        if (!mbar_wait(&k_full[s], (j / kKS) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        issue_s(tile_a, kd);
+        if (j > 0 && !issue_pv(tile_b, j - 1)) {
+          ok = false;
+          break;
+        }
+        issue_s(tile_b, kd);
+        tc_commit(&k_empty[s]);
       }
-      for (int t = 0; t < 2; ++t)
-        if (ok && n_tiles > 0) ok = issue_pv(t, n_tiles - 1);
+      if (ok && n_tiles > 0) ok = issue_pv(tile_a, n_tiles - 1) && issue_pv(tile_b, n_tiles - 1);
       tc_commit(o_final);
       if (!ok) atomicCAS(p.status, 0, kDevTimeout);
     }
@@ -357,6 +382,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       l *= alpha;
       if (need) m_used = m_new;
     }
+    if (t == 0 && (key0 + kKeys > n_valid_keys || loaded < kKeys)) {
+      // zero the V rows of keys that are not valid once the stage's copies
+      // have landed; both tiles' P V are issued after this tile's first P half
+      const int s = j % kVS;
+      if (!__all_sync(0xffffffffu, mbar_wait(&v_full[s], (j / kVS) & 1))) {
+        ok = false;
+        break;
+      }
+      uint8_t* vslot = base + C::kVOff + s * C::kSlotBytes;
+      for (int x = tid; x < kKeys * C::kHalves; x += kTileRows) {
+        const int c = x % kKeys, h = x / kKeys;
+        if (c >= loaded || key0 + c >= n_valid_keys) {
+#pragma unroll
+          for (int y = 0; y < 8; ++y)
+            *reinterpret_cast<uint4*>(vslot + h * C::kKVHalfBytes + c * 128 + y * 16) = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+      fence_proxy_async_smem();
+    }
     // P = 2^(s sl2 - m), two keys per packed f32x2 FMA / add, stored as bf16
     // pairs over this row's scores: the pairs of keys [64 hf, 64 hf + 64) go to
     // columns [32 hf, 32 hf + 32), whose scores have already been read
@@ -376,31 +420,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           pk[c / 2] = pack_bf16(a, b);
         }
         tmem_st32u(t_lane + hf * 32, pk);
+        tc_fence_before_sync();
+        mbar_arrive(&p_full[2 * t + hf]);
       }
       const float2 s = __fadd2_rn(__fadd2_rn(rs[0], rs[1]), __fadd2_rn(rs[2], rs[3]));
       l += s.x + s.y;
     }
-    if (t == 0 && (key0 + kKeys > n_valid_keys || loaded < kKeys)) {
-      // zero the V rows of keys that are not valid once the stage's copies
-      // have landed; both tiles' P V come after this tile's P is published
-      const int s = j % kVS;
-      if (!__all_sync(0xffffffffu, mbar_wait(&v_full[s], (j / kVS) & 1))) {
-        ok = false;
-        break;
-      }
-      uint8_t* vslot = base + C::kVOff + s * C::kSlotBytes;
-      for (int x = tid; x < kKeys * C::kHalves; x += kTileRows) {
-        const int c = x % kKeys, h = x / kKeys;
-        if (c >= loaded || key0 + c >= n_valid_keys) {
-#pragma unroll
-          for (int y = 0; y < 8; ++y)
-            *reinterpret_cast<uint4*>(vslot + h * C::kKVHalfBytes + c * 128 + y * 16) = make_uint4(0u, 0u, 0u, 0u);
-        }
-      }
-      fence_proxy_async_smem();
-    }
-    tc_fence_before_sync();
-    mbar_arrive(&p_full[t]);
   }
   if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0));
   tc_fence_after_sync();
