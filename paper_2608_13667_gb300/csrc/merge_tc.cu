@@ -16,19 +16,21 @@
 //               stage it reads its 128 scores, masks keys past the stage's
 //               pages and past its causal limit, keeps a running max raised
 //               only when a score exceeds it by more than 2^8 (O in TMEM is
-//               then rescaled in place), and writes P = 2^(s - m) as bf16 into
-//               TMEM over its own scores.  At the end it normalises O.
+//               then rescaled in place), and writes P = 2^(s - m) as two bf16
+//               terms (P_hi + P_lo, exact to about 16 bits) into TMEM over its
+//               own scores.  At the end it normalises O.
 //   warp 8      K loader, warp 9 V loader: page ids from the block table (32
 //               per read, one batch ahead), one 2 KiB TMA copy per (page,
 //               64-wide half of D) into separate K and V rings.
 //   warp 10     TMEM owner; lane 0 issues, per stage j and tile t = A, B,
-//                 O_t += P_t(j-1) V_{j-1}   (A = P from TMEM, M 128, N D)
+//                 O_t += P_t(j-1) V_{j-1}   (A = P_hi, P_lo from TMEM, M 128, N D)
 //                 S_t(j) = Q_t K_j^T        (M 128, N 128)
 //               so that the softmax of one tile overlaps the MMAs of the
 //               other.
 //
-// TMEM columns: tile t (0 = A, 1 = B) has S at 256 t (128 columns, P as bf16
-// pairs in its first 64) and O at 256 t + 128.  S_t(j + 1) overwrites P_t(j)
+// TMEM columns: tile t (0 = A, 1 = B) has S at 256 t (128 columns; the 16
+// columns of keys [16 k, 16 k + 16) then hold P_hi and P_lo of those keys as
+// bf16 pairs) and O at 256 t + 128.  S_t(j + 1) overwrites P_t(j)
 // only after O_t += P_t(j) V_j, which the same thread issued first; and the
 // commit that announces S_t(j) also covers O_t += P_t(j-1) V_{j-1}, so the
 // softmax may rescale O_t as soon as it sees S_t(j).
@@ -216,19 +218,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ---- MMA issuer ----------------------------------------------------------------
-  // One thread issues every MMA (two issuers interleaving on the tensor pipe
-  // measured slower).  It shares its sub-partition with two softmax warps, so
-  // the per-MMA work is kept to a constant add: a shared-memory descriptor's
-  // start field holds address / 16 (below 2^14 here), so the descriptor of an
-  // operand shifted by b bytes is the base descriptor + b / 16.
+  // One warp issues every MMA (two issuing warps interleaving on the tensor
+  // pipe measured slower): all its lanes run the loop with warp-uniform
+  // operands and an elected lane issues.  The issue rate bounds this kernel
+  // (tens of cycles per tcgen05.mma), so the per-MMA work is a constant add:
+  // a shared-memory descriptor's start field holds address / 16 (below 2^14
+  // here), so the descriptor of an operand shifted by b bytes is the base
+  // descriptor + b / 16.
   if (warp == kMmaWarp) {
-    if (lane == 0) {
+    {
       constexpr uint32_t idesc_s = tc_idesc_bf16(kTileRows, kKeys, 0, 0);
       constexpr uint32_t idesc_o = tc_idesc_bf16(kTileRows, D, 0, 1);
       const uint64_t q_desc = tc_desc_sw128(smem_addr(base + C::kQOff), 16, 1024);
       const uint64_t k_desc0 = tc_desc_sw128(smem_addr(base + C::kKOff), 16, 1024);
       const uint64_t v_desc0 = tc_desc_sw128(smem_addr(base + C::kVOff), C::kKVHalfBytes, 1024);
-      bool ok = mbar_wait(q_ready, 0);
+      bool ok = __all_sync(0xffffffffu, mbar_wait(q_ready, 0));
       tc_fence_after_sync();
       // O_t += P_t(i) V_i, P_t(i) read from TMEM over S_t(i); each half of P
       // (64 keys) is published on its own, so the first half's MMAs run while
@@ -236,21 +240,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue_pv = [&](auto tile, int i) -> bool {
         constexpr int t = decltype(tile)::value;
         const int s = i % kVS;
-        if (t == 0 && !mbar_wait(&v_full[s], (i / kVS) & 1)) return false;
+        if (t == 0 && !__all_sync(0xffffffffu, mbar_wait(&v_full[s], (i / kVS) & 1))) return false;
         const uint64_t vd = v_desc0 + (uint64_t)((s * C::kSlotBytes) >> 4);
         const uint32_t acc0 = i > 0 ? 1u : 0u;
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
-          if (!mbar_wait(&p_full[2 * t + hf], i & 1)) return false;
+          if (!__all_sync(0xffffffffu, mbar_wait(&p_full[2 * t + hf], i & 1))) return false;
           tc_fence_after_sync();
 #pragma unroll
           for (int kq = 0; kq < kKeys / 32; ++kq) {
             const int ks = hf * (kKeys / 32) + kq;
-            tc_mma_bf16_tmem_a(tmem + t * kTmemTile + kTmemO, tmem + t * kTmemTile + ks * 8,
-                               vd + (uint64_t)((ks * 16 * 128) >> 4), idesc_o, ks > 0 ? 1u : acc0);
+            const uint64_t vk = vd + (uint64_t)((ks * 16 * 128) >> 4);
+            tc_mma_bf16_tmem_a_elect(tmem + t * kTmemTile + kTmemO, tmem + t * kTmemTile + ks * 16, vk, idesc_o,
+                               ks > 0 ? 1u : acc0);                                    // P_hi
+            tc_mma_bf16_tmem_a_elect(tmem + t * kTmemTile + kTmemO, tmem + t * kTmemTile + ks * 16 + 8, vk, idesc_o,
+                               1u);                                                     // P_lo
           }
         }
-        if (t == 1) tc_commit(&v_empty[s]);
+        if (t == 1) tc_commit_elect(&v_empty[s]);
         return true;
       };
       // S_t(j) = Q_t K_j^T
@@ -260,10 +267,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int h = 0; h < C::kHalves; ++h)
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
-            tc_mma_bf16(tmem + t * kTmemTile,
+            tc_mma_bf16_elect(tmem + t * kTmemTile,
                         q_desc + (uint64_t)((t * C::kQTileBytes + h * C::kQHalfBytes + kk * 32) >> 4),
                         kd + (uint64_t)((h * C::kKVHalfBytes + kk * 32) >> 4), idesc_s, (h | kk) != 0);
-        tc_commit(&s_full[t]);
+        tc_commit_elect(&s_full[t]);
       };
       const std::integral_constant<int, 0> tile_a;
       const std::integral_constant<int, 1> tile_b;
@@ -274,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        if (!mbar_wait(&k_full[s], (j / kKS) & 1)) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&k_full[s], (j / kKS) & 1))) {
           ok = false;
           break;
         }
@@ -285,11 +292,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         issue_s(tile_b, kd);
-        tc_commit(&k_empty[s]);
+        tc_commit_elect(&k_empty[s]);
       }
       if (ok && n_tiles > 0) ok = issue_pv(tile_a, n_tiles - 1) && issue_pv(tile_b, n_tiles - 1);
-      tc_commit(o_final);
-      if (!ok) atomicCAS(p.status, 0, kDevTimeout);
+      tc_commit_elect(o_final);
+      if (!ok && lane == 0) atomicCAS(p.status, 0, kDevTimeout);
     }
     __syncwarp();
     named_barrier_sync(1, kSoftThreads + 32);
@@ -401,9 +408,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       fence_proxy_async_smem();
     }
-    // P = 2^(s sl2 - m), two keys per packed f32x2 FMA / add, stored as bf16
-    // pairs over this row's scores: the pairs of keys [64 hf, 64 hf + 64) go to
-    // columns [32 hf, 32 hf + 32), whose scores have already been read
+    // P = 2^(s sl2 - m) (two keys per packed f32x2 FMA / add) as two bf16
+    // terms, P_hi = bf16(P) and P_lo = bf16(P - P_hi), so that P V is exact to
+    // about 16 bits whatever the spread of the scores.  The 16 score columns
+    // of keys [16 ks, 16 ks + 16) take P_hi of those keys (8 columns of bf16
+    // pairs) and then P_lo (8 columns): each store overwrites only scores
+    // already read.
     {
       const float2 scale2 = make_float2(sl2, sl2), neg_m2 = make_float2(-m_used, -m_used);
       float2 rs[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
@@ -411,15 +421,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int hf = 0; hf < 2; ++hf) {
         float sc[64];
         load_half(hf, sc);
-        uint32_t pk[32];
 #pragma unroll
-        for (int c = 0; c < 64; c += 2) {
-          const float2 x = __ffma2_rn(make_float2(sc[c], sc[c + 1]), scale2, neg_m2);
-          const float a = ex2(x.x), b = ex2(x.y);
-          rs[(c >> 1) & 3] = __fadd2_rn(rs[(c >> 1) & 3], make_float2(a, b));
-          pk[c / 2] = pack_bf16(a, b);
+        for (int kq = 0; kq < 4; ++kq) {  // 16 keys per step
+          uint32_t pk[16];
+#pragma unroll
+          for (int c = 0; c < 16; c += 2) {
+            const float2 x = __ffma2_rn(make_float2(sc[kq * 16 + c], sc[kq * 16 + c + 1]), scale2, neg_m2);
+            const float a = ex2(x.x), b = ex2(x.y);
+            rs[(c >> 1) & 3] = __fadd2_rn(rs[(c >> 1) & 3], make_float2(a, b));
+            const uint32_t hi = pack_bf16(a, b);
+            pk[c / 2] = hi;
+            pk[8 + c / 2] = pack_bf16(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
+          }
+          tmem_st16u_nowait(t_lane + (hf * 4 + kq) * 16, pk);
         }
-        tmem_st32u(t_lane + hf * 32, pk);
+        tmem_wait_st();
         tc_fence_before_sync();
         mbar_arrive(&p_full[2 * t + hf]);
       }

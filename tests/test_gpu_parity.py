@@ -277,6 +277,52 @@ def test_merge_prefill(stlib, D, Hq, Hkv, L0, T):
     compare(o[0], lse[0], o_ref, l_ref, "sibling after merge")
 
 
+@pytest.mark.parametrize("D,Hq,Hkv,L0,T", [
+    (128, 32, 8, 2047, 1),      # 2048 keys: the last merge on the two-term path
+    (128, 32, 8, 2048, 1),      # 2049 keys: the first on the paired-tile path
+    (64, 8, 2, 2100, 64),       # D 64, one CTA, tile B partly filled
+    (128, 32, 8, 2500, 37),     # 148 stacked rows: tile B ragged
+    (128, 64, 8, 3001, 40),     # 320 rows: a second CTA, context ends mid-page
+    (128, 8, 8, 4096, 300),     # G 1, page-aligned context
+    (64, 32, 4, 5000, 129),     # short last stage (few pages loaded)
+])
+def test_merge_prefill_long_context(stlib, D, Hq, Hkv, L0, T):
+    w = _small(D, Hq, Hkv, n_blocks=1024, L=2)
+    run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=8)
+    m = run.create()
+    run.append([m], L0, ("ctx",))
+    qm, om, lm, L0r = run.merge(m, T, ("merge",))
+    assert L0r == L0
+    run.pool.sync()
+    run.check_tables()
+    for layer in range(2):
+        k, v = run.context(m, layer)
+        o_ref, l_ref = A.merge_prefill(qm[layer].cpu(), k, v, L0)
+        compare(om[layer], lm[layer], o_ref, l_ref, f"long merge layer {layer}")
+
+
+@pytest.mark.parametrize("D,kind", [(128, "merge"), (64, "merge"), (128, "decode"), (64, "decode")])
+def test_running_max_raised_after_the_first_stage(stlib, D, kind):
+    # values x3: scores have a standard deviation near 9, so later stages keep
+    # exceeding the running max by more than 2^8 and O is rescaled in TMEM
+    w = _small(D, 16, 4, n_blocks=1024, L=1, scale=3.0)
+    run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=8)
+    m = run.create()
+    run.append([m], 6000, ("ctx",))
+    if kind == "merge":
+        qm, om, lm, L0 = run.merge(m, 50, ("merge",))
+        k, v = run.context(m, 0)
+        o_ref, l_ref = A.merge_prefill(qm[0].cpu(), k, v, L0)
+        compare(om[0], lm[0], o_ref, l_ref, "merge with rescales")
+    else:
+        aux = run.fork(m, 2)
+        br = [m] + aux
+        run.append(br, 1, ("s",))
+        q, o, lse = run.decode(br, ("q",))
+        o_ref, l_ref = run.oracle_decode(br, q, 0)
+        compare(o[0], lse[0], o_ref, l_ref, "decode with rescales")
+
+
 def test_merge_of_one_row_equals_decode_after_append(stlib):
     w = _small(128, 32, 8, n_blocks=256, L=1)
     run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=8)
