@@ -1,5 +1,5 @@
-// Paged attention on the 5th-generation tensor cores (tcgen05, accumulators
-// in tensor memory): fork-group decode partials and the merge prefill.
+// Fork-group decode partials on the 5th-generation tensor cores (tcgen05,
+// accumulators in tensor memory).  The merge prefill is in merge_tc.cu.
 //
 // Section 3.3 of the paper: every branch receives the snapshot H_t + R_t, so
 // the prefix KV is shared by all decoding streams; Section 4.4: branch load
@@ -7,26 +7,26 @@
 // pages of one KV head of one layer and stacks every query row that reads
 // it -- for a shared prefix all branches of the fork group x the G query
 // heads of the KV head (<= 48 rows) -- so each prefix page crosses HBM once
-// per group.  Section 3.5: the merged thoughts are appended after main's
-// context and read in order, so a merge CTA stacks 128 (thought row, head)
-// rows and walks main's pages up to its causal limit (row i sees keys
-// [0, L0 + i]).
+// per group.
 //
 // CTA layout (192 threads, 2 CTAs per SM):
-//   warps 0..3  softmax (only ceil(rows/32) of them run): thread r owns query
-//               row r = TMEM lane r.  It loads its Q row into shared memory;
-//               per stage it reads its scores from TMEM, masks keys past the
-//               run (and past its causal limit in the merge), keeps a running
-//               max that is raised only when a score exceeds it by more than
-//               2^8 (O in TMEM is then rescaled in place), and writes
-//               P = 2^(s - m) as bf16 over the stage's consumed K slot.  At the
-//               end it normalises O out of TMEM (decode: a split-KV partial
-//               with its log-sum-exp; merge: the final row).
+//   warps 0..3  softmax (only ceil(rows/16) of them run).  The MMA is
+//               M = 64: row r sits in TMEM lane 32 (r / 16) + r % 16, and
+//               threads t and t + 16 of a warp share row t, each with half of
+//               the stage's keys and half of the O columns (16-lane TMEM
+//               loads with a column split).  A thread loads its half of its
+//               Q row into shared memory; per stage it reads its scores from
+//               TMEM, masks keys past the run, keeps a running max (combined
+//               with its partner by one shuffle) that is raised only when a
+//               score exceeds it by more than 2^8 (O in TMEM is then rescaled
+//               in place), and writes P = 2^(s - m) as two bf16 terms over the
+//               stage's consumed K slot.  At the end it normalises O out of
+//               TMEM: a split-KV partial with its log-sum-exp.
 //   warp 4      loader: page ids from the block table (32 per read, one batch
 //               ahead), one 2 KiB TMA copy per (page, 64-wide half of D, K|V)
 //               into a ring of stages, per-stage mbarriers with byte counts.
-//   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M=128, N=64 keys)
-//               and O += P V (M=128, N=D) and commits them to mbarriers.  S is
+//   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M=64, N=64 keys)
+//               and O += P V (M=64, N=D) and commits them to mbarriers.  S is
 //               double-buffered in TMEM: S_{j+1} is issued before P_j V_j when
 //               its data has landed, so the softmax of stage j+1 overlaps the
 //               tensor work of stage j.
@@ -35,13 +35,13 @@
 // Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
 //   Q  [D/64][rows][64]       K-major A (SBO 1024)
 //   K  [D/64][keys][64]       K-major B (SBO 1024)
-//   P  [rows][keys]           K-major A (SBO 1024), written over K (decode:
-//                             two bf16 terms P_hi, P_lo, one after the other)
+//   P  [rows][keys]           K-major A (SBO 1024), written over K: two bf16
+//                             terms P_hi, P_lo, one after the other
 //   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
-// The MMA always computes 128 rows.  In decode only the first <= 48 Q and P
-// rows are written; rows past them read whatever follows in shared memory and
-// only produce accumulator rows that nobody reads (each output row depends
-// on its own A row only).  V rows of keys that are not valid (past the run,
+// The MMA computes 64 rows and only the first <= 48 Q and P rows are
+// written; rows past them read whatever follows in shared memory and only
+// produce accumulator rows that nobody reads (each output row depends on its
+// own A row only).  V rows of keys that are not valid (past the run,
 // or in pages a short last stage did not load) are zeroed before P V, so
 // stale shared or pool memory cannot turn 0 * x into NaN in a real row.
 #include <math.h>
@@ -53,7 +53,6 @@ namespace st {
 
 namespace {
 
-constexpr int kMmaRows = 128;
 constexpr int kLoadWarp = 4, kMmaWarp = 5;
 constexpr int kThreads = 6 * 32;
 constexpr uint32_t kTmemCols = 256;
@@ -64,29 +63,26 @@ constexpr int kMaxDevices = 64;
 
 constexpr int cmax(int a, int b) { return a > b ? a : b; }
 
-template <int D, bool kDecode, bool kSplit = kDecode>
+template <int D>
 struct TcCfg {
   static constexpr int kHalves = D / 64;
   static constexpr int kKeys = 64;                     // keys per stage
   static constexpr int kPagesPerStage = kKeys / kPageTokens;
-  static constexpr int kStages = kDecode ? 3 : 2;
-  // MMA M: decode stacks <= 48 rows and uses M = 64, whose accumulator rows
-  // sit in TMEM lanes 0..15 of each warp's 32-lane quarter (row r at lane
-  // 32 * (r / 16) + r % 16); the merge uses M = 128 (row r at lane r).
-  static constexpr int kM = kDecode ? 64 : 128;
+  static constexpr int kStages = 3;
+  // MMA M = 64 for <= 48 stacked rows: accumulator rows sit in TMEM lanes
+  // 0..15 of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16)
+  static constexpr int kM = 64;
   static constexpr int kRowsPerWarp = kM / 4;
-  static constexpr int kQRows = kDecode ? 48 : 128;    // Q/P rows stored
+  static constexpr int kQRows = 48;                    // Q/P rows stored
   static constexpr int kQHalfBytes = kQRows * 128;
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kKVHalfBytes = kKeys * 128;
-  // P as two bf16 terms (P = P_hi + P_lo, two MMAs against the same V): with
-  // few keys the rounding of a single bf16 P does not average out.  Decode
-  // always splits; the merge splits only when its rows see few keys (the
-  // second term costs it a second CTA per SM).
-  static constexpr bool kSplitP = kSplit;
+  // P as two bf16 terms (P = P_hi + P_lo, two MMAs against the same V): the
+  // rounding of a single bf16 P does not average out when a row sees few
+  // keys or its weights are peaked
   static constexpr int kPTermBytes = kQRows * 128;                // one term, kQRows rows
-  static constexpr int kPloOffset = kSplitP ? kPTermBytes : 0;    // P_lo after P_hi in the K slot
-  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, (kSplitP ? 2 : 1) * kPTermBytes);
+  static constexpr int kPloOffset = kPTermBytes;                  // P_lo after P_hi in the K slot
+  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, 2 * kPTermBytes);
   static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
   static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
@@ -97,11 +93,11 @@ struct TcCfg {
   static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 };
 
-template <int D, bool kDecode, bool kSplit>
+template <int D>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
-  using C = TcCfg<D, kDecode, kSplit>;
+  using C = TcCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
@@ -124,28 +120,13 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int G = p.G;
 
   // ---- what this CTA reads and for whom ------------------------------------------
-  int slot, page_begin, n_pages, n_valid_keys, n_rows, min_limit, row_base = 0;
-  AttnItem item{};
   const int32_t* members = p.members ? p.members : inl.members;
-  if (kDecode) {
-    item = p.items ? p.items[blockIdx.x] : inl.items[blockIdx.x];
-    slot = item.slot;
-    page_begin = item.page_begin;
-    n_pages = item.n_pages;
-    n_valid_keys = item.n_tokens;
-    n_rows = item.n_members * G;
-    min_limit = item.n_tokens;
-  } else {
-    slot = p.slot;
-    page_begin = 0;
-    row_base = blockIdx.x * kMmaRows;
-    n_rows = min(kMmaRows, p.T * G - row_base);
-    const int t_first = row_base / G;
-    const int t_last = (row_base + n_rows - 1) / G;
-    n_pages = (p.L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
-    n_valid_keys = p.L0 + p.T;
-    min_limit = p.L0 + t_first + 1;
-  }
+  const AttnItem item = p.items ? p.items[blockIdx.x] : inl.items[blockIdx.x];
+  const int slot = item.slot;
+  const int page_begin = item.page_begin;
+  const int n_pages = item.n_pages;
+  const int n_valid_keys = item.n_tokens;
+  const int n_rows = item.n_members * G;
   const int n_tiles = (n_pages + C::kPagesPerStage - 1) / C::kPagesPerStage;
   const int n_sw = (n_rows + C::kRowsPerWarp - 1) / C::kRowsPerWarp;  // softmax warps with rows
   const int n_swt = n_sw * 32;
@@ -177,9 +158,8 @@ __global__ void __launch_bounds__(kThreads, 2)
       prefetch_tensormap(&kmap);
       prefetch_tensormap(&vmap);
     }
-    // decode streams every page once; the merge's CTAs of one (layer, head)
-    // all walk the same pages
-    const uint64_t policy = kDecode ? l2_policy_evict_first() : l2_policy_evict_last();
+    // every page is streamed once
+    const uint64_t policy = l2_policy_evict_first();
     const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
@@ -289,12 +269,10 @@ __global__ void __launch_bounds__(kThreads, 2)
           tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + ks * 32, 16, 1024),
                       tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
                       (j > 0 || ks > 0) ? 1u : 0u);
-        if constexpr (C::kSplitP) {
 #pragma unroll
-          for (int ks = 0; ks < C::kKeys / 16; ++ks)
-            tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
-                        tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
-        }
+        for (int ks = 0; ks < C::kKeys / 16; ++ks)
+          tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
+                      tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
         tc_commit(&empty[s]);
         tc_commit(o_ready);
         if (jn < n_tiles && !early && !issue_s(jn)) {
@@ -314,34 +292,23 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (warp >= n_sw) return;
 
   // ---- softmax warps ---------------------------------------------------------------
-  // Merge (M = 128): thread r owns row r (TMEM lane r), all of its keys and O
-  // columns.  Decode (M = 64): the rows sit in lanes 0..15 of each warp's
-  // quarter and threads t and t + 16 share row t: half of the stage's keys
-  // and half of the O columns each (16-lane TMEM loads with a column split),
-  // the row max and sum combined with one shuffle.
-  constexpr bool kPair = C::kM == 64;
-  constexpr int kKpt = C::kKeys / (kPair ? 2 : 1);  // keys per thread per stage
-  constexpr int kOpt = D / (kPair ? 2 : 1);         // O columns per thread
-  const int tid = threadIdx.x;                      // 0 .. n_swt-1, for cooperative loops
-  const int half = kPair ? (lane >> 4) : 0;
-  const int r = kPair ? warp * 16 + (lane & 15) : threadIdx.x;  // this thread's row
+  // Threads t and t + 16 of a warp share row t: half of the stage's keys and
+  // half of the O columns each, the row max and sum combined with one shuffle.
+  constexpr int kKpt = C::kKeys / 2;  // keys per thread per stage
+  constexpr int kOpt = D / 2;         // O columns per thread
+  const int tid = threadIdx.x;        // 0 .. n_swt-1, for cooperative loops
+  const int half = lane >> 4;
+  const int r = warp * 16 + (lane & 15);  // this thread's row
   const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
   const bool valid = r < n_rows;
   int qrow = 0, head = 0;
   if (valid) {
-    if (kDecode) {
-      qrow = members[item.member_base + r / G];
-      head = kvh * G + r % G;
-    } else {
-      const int gr = row_base + r;
-      qrow = gr / G;
-      head = kvh * G + gr % G;
-    }
+    qrow = members[item.member_base + r / G];
+    head = kvh * G + r % G;
   }
-  const int limit = (!kDecode && valid) ? p.L0 + qrow + 1 : n_valid_keys;
   if (r < C::kQRows) {
     const uint4* src = reinterpret_cast<const uint4*>(p.q + (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * D);
-    constexpr int kChunks = D / 8 / (kPair ? 2 : 1);  // 16-byte chunks of the row this thread writes
+    constexpr int kChunks = D / 16;  // 16-byte chunks of the half row this thread writes
 #pragma unroll
     for (int cc = 0; cc < kChunks; ++cc) {
       const int c = half * kChunks + cc;
@@ -353,14 +320,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   mbar_arrive(q_ready);
 
   // this thread's 32-column pieces of its O row: [o_col(k), o_col(k) + 32)
-  auto o_load = [&](int k, float* o) {
-    if constexpr (kPair) tmem_ld16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
-    else tmem_ld32(t_lane + kTmemO + k * 32, o);
-  };
-  auto o_store = [&](int k, const float* o) {
-    if constexpr (kPair) tmem_st16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
-    else tmem_st32(t_lane + kTmemO + k * 32, o);
-  };
+  auto o_load = [&](int k, float* o) { tmem_ld16x2_32<D / 2>(t_lane + kTmemO + k * 32, o); };
+  auto o_store = [&](int k, const float* o) { tmem_st16x2_32<D / 2>(t_lane + kTmemO + k * 32, o); };
   auto o_col = [&](int k) { return half * (D / 2) + k * 32; };
 
   const float sl2 = p.scale_log2;
@@ -377,17 +338,15 @@ __global__ void __launch_bounds__(kThreads, 2)
     // domain, x = s * sl2
     float sc[kKpt];
     static_assert(C::kKeys == 64, "64 keys per stage");
-    if constexpr (kPair) tmem_ld16x2_32<32>(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
-    else tmem_ld64(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
+    tmem_ld16x2_32<32>(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
     const int key0 = j * C::kKeys;
     const int kbase = half * kKpt;  // this thread's first key within the stage
     const int np = min(C::kPagesPerStage, n_pages - j * C::kPagesPerStage);
     const int loaded = np * kPageTokens;
-    const bool edge = key0 + C::kKeys > min_limit || loaded < C::kKeys;
-    if (edge) {
+    if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
 #pragma unroll
       for (int c = 0; c < kKpt; ++c)
-        if (kbase + c >= loaded || key0 + kbase + c >= limit) sc[c] = -INFINITY;
+        if (kbase + c >= loaded || key0 + kbase + c >= n_valid_keys) sc[c] = -INFINITY;
     }
     // 8 independent max chains, then a tree (short dependency chains)
     float mx8[8];
@@ -397,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int c = 8; c < kKpt; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sc[c]);
     float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                      fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-    if constexpr (kPair) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
     const float m_new = fmaxf(m_used, mx * sl2);  // sl2 > 0: max commutes with the scale
     const bool need = valid && m_new > m_used + kRescaleThreshold;
     if (__any_sync(0xffffffffu, need)) {
@@ -425,7 +384,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint8_t* kslot = ring + s * C::kStageBytes;  // S_j has been consumed: P_j goes over K_j
     if (valid) {
       uint32_t pk[kKpt / 2];
-      uint32_t pl[C::kSplitP ? kKpt / 2 : 1];
+      uint32_t pl[kKpt / 2];
       float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < kKpt; c += 2) {
@@ -433,8 +392,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         rs[(c >> 1) & 7] += a + b;
         const uint32_t hi = pack_bf16(a, b);
         pk[c / 2] = hi;
-        if constexpr (C::kSplitP)  // remainders below the bf16 rounding of a and b
-          pl[c / 2] = pack_bf16(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
+        // remainders below the bf16 rounding of a and b
+        pl[c / 2] = pack_bf16(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
       }
       l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
 #pragma unroll
@@ -442,9 +401,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int c = half * (kKpt / 8) + cc;  // 16-byte chunk of the P row (8 keys)
         const uint32_t off = r * 128 + ((c ^ (r & 7)) << 4);
         *reinterpret_cast<uint4*>(kslot + off) = make_uint4(pk[4 * cc], pk[4 * cc + 1], pk[4 * cc + 2], pk[4 * cc + 3]);
-        if constexpr (C::kSplitP)
-          *reinterpret_cast<uint4*>(kslot + C::kPloOffset + off) =
-              make_uint4(pl[4 * cc], pl[4 * cc + 1], pl[4 * cc + 2], pl[4 * cc + 3]);
+        *reinterpret_cast<uint4*>(kslot + C::kPloOffset + off) =
+            make_uint4(pl[4 * cc], pl[4 * cc + 1], pl[4 * cc + 2], pl[4 * cc + 3]);
       }
     }
     if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
@@ -468,16 +426,12 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0));
   tc_fence_after_sync();
   if (ok) {
-    if constexpr (kPair) l += __shfl_xor_sync(0xffffffffu, l, 16);  // the row's full sum
+    l += __shfl_xor_sync(0xffffffffu, l, 16);  // the row's full sum
     const float inv = 1.f / l;
     float* dst = nullptr;
     float* dst_lse = nullptr;
     if (valid) {
-      int64_t idx;
-      if (kDecode)
-        idx = (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * p.max_splits + item.split;
-      else
-        idx = ((int64_t)layer * p.T + qrow) * p.Hq + head;
+      const int64_t idx = (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * p.max_splits + item.split;
       dst = p.out_o + idx * D;
       if (half == 0) dst_lse = p.out_lse + idx;
     }
@@ -500,10 +454,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   named_barrier_sync(1, n_swt + 32);
 }
 
-template <int D, bool kDecode, bool kSplit>
+template <int D>
 cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
                         const InlineDecodePlan& inl, int n_ctas, cudaStream_t s) {
-  using C = TcCfg<D, kDecode, kSplit>;
+  using C = TcCfg<D>;
   // the shared-memory opt-in is a per-device function attribute
   static bool configured[kMaxDevices] = {};
   int dev = 0;
@@ -511,31 +465,27 @@ cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const Attn
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    e = cudaFuncSetAttribute(attend_tc_kernel<D, kDecode, kSplit>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             C::kSmemBytes);
+    e = cudaFuncSetAttribute(attend_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  attend_tc_kernel<D, kDecode, kSplit><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
+  attend_tc_kernel<D><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
   return cudaGetLastError();
 }
 
 template <int D>
 int decode_ctas_per_sm_t() {
-  using C = TcCfg<D, true>;
-  if (cudaFuncSetAttribute(attend_tc_kernel<D, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           C::kSmemBytes) != cudaSuccess)
+  using C = TcCfg<D>;
+  if (cudaFuncSetAttribute(attend_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+      cudaSuccess)
     return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, true, true>, kThreads,
-                                                    C::kSmemBytes) != cudaSuccess)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D>, kThreads, C::kSmemBytes) !=
+      cudaSuccess)
     return 0;
   return n < 2 ? n : 2;  // two CTAs' TMEM (2 x 256 columns) fill an SM
 }
-
-// Merges whose longest row sees at most this many keys use two P terms.
-constexpr int kMergeSplitMaxKeys = 2048;
 
 }  // namespace
 
@@ -544,20 +494,8 @@ cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const
   static const InlineDecodePlan kNone{};
   const InlineDecodePlan& ip = inl ? *inl : kNone;
   if (n_items <= 0) return cudaSuccess;
-  if (D == 128) return launch_tc_t<128, true, true>(km, vm, p, ip, n_items, s);
-  if (D == 64) return launch_tc_t<64, true, true>(km, vm, p, ip, n_items, s);
-  return cudaErrorInvalidValue;
-}
-
-cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int D,
-                            cudaStream_t s) {
-  static const InlineDecodePlan kNone{};
-  if (p.T <= 0) return cudaSuccess;
-  // long contexts: two query tiles per CTA sharing K/V (merge_tc.cu)
-  if ((int64_t)p.L0 + p.T > kMergeSplitMaxKeys) return launch_merge_pair(km, vm, p, D, s);
-  const int n_tiles = (p.T * p.G + kMmaRows - 1) / kMmaRows;
-  if (D == 128) return launch_tc_t<128, false, true>(km, vm, p, kNone, n_tiles, s);
-  if (D == 64) return launch_tc_t<64, false, true>(km, vm, p, kNone, n_tiles, s);
+  if (D == 128) return launch_tc_t<128>(km, vm, p, ip, n_items, s);
+  if (D == 64) return launch_tc_t<64>(km, vm, p, ip, n_items, s);
   return cudaErrorInvalidValue;
 }
 

@@ -2,8 +2,7 @@
 //
 //   table_update  -- refresh rows of the device block tables from the host's
 //   append_kv     -- copy-on-write page copies + scatter of new K/V rows
-//   attend_tc     -- paged decode partials and short causal merge prefills
-//                    (tcgen05, TMEM accumulators)
+//   attend_tc     -- paged decode partials (tcgen05, TMEM accumulators)
 //   merge_pair    -- causal merge prefill, two query tiles per CTA (tcgen05)
 //   lse_combine   -- log-sum-exp combine of decode partials
 #pragma once
@@ -115,14 +114,10 @@ cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, 
 // Decode partials on tcgen05 (one CTA per item x KV head x layer).
 cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
                              const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s);
-// Causal merge prefill on tcgen05 (p.slot, p.L0, p.T, p.q -> p.out_o, p.out_lse):
-// contexts of at most 2048 keys on attend_tc (two P terms), longer ones on
-// launch_merge_pair.
+// Causal merge prefill on tcgen05 (p.slot, p.L0, p.T, p.q -> p.out_o, p.out_lse),
+// two 128-row query tiles per CTA sharing K/V (merge_tc.cu).
 cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int D,
                             cudaStream_t s);
-// The same prefill with two 128-row query tiles per CTA sharing K/V (merge_tc.cu).
-cudaError_t launch_merge_pair(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int D,
-                              cudaStream_t s);
 // CTAs of the tcgen05 decode kernel resident per SM (0 on error).
 int decode_tc_ctas_per_sm(int D);
 

@@ -488,8 +488,8 @@ cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const At
 
 }  // namespace
 
-cudaError_t launch_merge_pair(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int D,
-                              cudaStream_t s) {
+cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int D,
+                            cudaStream_t s) {
   if (p.T <= 0) return cudaSuccess;
   if (D == 128) return launch_pair_t<128>(km, vm, p, s);
   if (D == 64) return launch_pair_t<64>(km, vm, p, s);
