@@ -178,11 +178,23 @@ def build_long_workload(w, dev):
     return pool, branches
 
 
+def _workload(args):
+    """The bench workload: config N, or the long-trajectory one with another
+    branch count (--n-aux)."""
+    from workloads import get
+    from workloads.configs import long_with_branches
+    if args.n_aux is None:
+        return get(args.config)
+    if args.config != 4:
+        raise SystemExit("--n-aux applies to config 4 (long trajectory)")
+    return long_with_branches(args.n_aux)
+
+
 def run_ours(args, rank, ws, local):
     import torch
     import paper_2608_13667_gb300 as st
-    from workloads import get, kv_rows, queries
-    w = get(args.config)
+    from workloads import kv_rows, queries
+    w = _workload(args)
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     st.build()
@@ -438,7 +450,7 @@ def run_cycle():
 # --------------------------------------------------------------------------- oracle
 
 def oracle_sample_step(w, dev, layer, task=0):
-    """The float64 oracle over one layer of one fork group (5 branches): a
+    """The float64 oracle over one layer of one fork group (all its branches): a
     bounded sample of the step.  Returns (seconds of oracle work, branch-steps)."""
     import torch
     from oracle import attention as A
@@ -468,14 +480,13 @@ def oracle_sample_step(w, dev, layer, task=0):
 def cpu_baseline(w, dev):
     dt, units = oracle_sample_step(w, dev, layer=0)
     return {"value": units / dt, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"1 of {w.n_layers} layers of 1 of {w.n_tasks} fork groups (5 branches, "
+            "sample": f"1 of {w.n_layers} layers of 1 of {w.n_tasks} fork groups ({w.n_aux + 1} branches, "
                       f"{w.prefix[0]}-token prefix), float64 numpy; {dt:.1f} s"}
 
 
 def run_reference(args, rank, ws, local):
     import torch
-    from workloads import get
-    w = get(args.config)
+    w = _workload(args)
     if rank != 0:
         return {}
     dev = torch.device("cuda", local) if torch.cuda.is_available() else torch.device("cpu")
@@ -487,7 +498,7 @@ def run_reference(args, rank, ws, local):
         total_dt += dt
         total_units += units
     value = total_units / total_dt
-    sample = (f"each step: 1 layer of 1 fork group (5 branches, {w.prefix[0]}-token prefix) "
+    sample = (f"each step: 1 layer of 1 fork group ({w.n_aux + 1} branches, {w.prefix[0]}-token prefix) "
               f"of the {w.name} workload, float64 numpy oracle")
     return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_dt / args.steps * 1e3,
@@ -506,6 +517,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--n-aux", type=int, default=None,
+                    help="config 4 with this many auxiliary branches per group instead of 4")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-small", action="store_true",
                     help="run the small decode + merge case used for ncu captures and exit")
@@ -530,8 +543,7 @@ def main():
         res = run_ours(args, rank, ws, local)
         if rank == 0 and ws == 1 and not args.no_cpu_baseline:
             import torch
-            from workloads import get
-            res["cpu_baseline"] = cpu_baseline(get(args.config), torch.device("cuda", local))
+            res["cpu_baseline"] = cpu_baseline(_workload(args), torch.device("cuda", local))
     if rank == 0:
         print(json.dumps(res), flush=True)
     if ws > 1:

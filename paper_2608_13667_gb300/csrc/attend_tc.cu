@@ -7,7 +7,10 @@
 // pages of one KV head of one layer and stacks every query row that reads
 // it -- for a shared prefix all branches of the fork group x the G query
 // heads of the KV head (<= 48 rows) -- so each prefix page crosses HBM once
-// per group.
+// per group.  A group with more than 48 stacked rows (more than 48 / G
+// branches; Section 3.2 lets the branch count vary) is split into subgroups
+// whose items over the same pages run next to each other, so the second
+// read of a page comes from L2.
 //
 // CTA layout (192 threads, 2 CTAs per SM):
 //   warps 0..3  softmax (only ceil(rows/16) of them run).  The MMA is
@@ -158,8 +161,9 @@ __global__ void __launch_bounds__(kThreads, 2)
       prefetch_tensormap(&kmap);
       prefetch_tensormap(&vmap);
     }
-    // every page is streamed once
-    const uint64_t policy = l2_policy_evict_first();
+    // a page is streamed once, unless a sibling item (the group's other
+    // subgroup, scheduled next to this one) reads it too: then keep it in L2
+    const uint64_t policy = item.reread ? l2_policy_evict_normal() : l2_policy_evict_first();
     const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;

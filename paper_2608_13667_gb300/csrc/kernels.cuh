@@ -61,7 +61,7 @@ struct AttnItem {
   int32_t member_base; // index of the first member in the members array
   int32_t n_members;
   int32_t split;       // partial slot this item writes
-  int32_t pad;
+  int32_t reread;      // 1: a sibling item (another subgroup of the fork group) reads the same pages
 };
 
 struct AttnParams {

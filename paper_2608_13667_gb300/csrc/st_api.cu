@@ -15,6 +15,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <tuple>
 #include <new>
 #include <string>
 #include <vector>
@@ -602,7 +603,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
 
   // ---- group by fork family, find the shared full pages --------------------
   std::vector<int32_t> shared(n_br, 0);   // pages of branch i read through its group
-  struct Group { std::vector<int> members; int32_t pages; };
+  struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split; };
   std::vector<Group> groups;
   {
     std::map<int32_t, std::vector<int>> fam;
@@ -615,22 +616,34 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     const int per_group = std::max(1, kMaxAttnRows / G);
     for (int32_t f : order) {
       const std::vector<int>& mem = fam[f];
-      for (size_t b0 = 0; b0 < mem.size(); b0 += per_group) {
-        const size_t b1 = std::min(mem.size(), b0 + per_group);
-        if (b1 - b0 < 2) continue;
+      // full pages held by every member of mem[b0, b1)
+      auto common_pages = [&](size_t b0, size_t b1) {
         const SeqSlot& lead = bp.slot(slots[mem[b0]]);
         int64_t min_len = lead.len;
         int32_t pages = (int32_t)lead.table.size();
-        for (size_t m = b0 + 1; m < b1; ++m) {
-          const SeqSlot& ss = bp.slot(slots[mem[m]]);
+        for (size_t x = b0 + 1; x < b1; ++x) {
+          const SeqSlot& ss = bp.slot(slots[mem[x]]);
           pages = std::min(pages, lcp_pages(lead.table, ss.table));
           min_len = std::min<int64_t>(min_len, ss.len);
         }
-        pages = std::min<int32_t>(pages, (int32_t)(min_len / kPageTokens));
+        return std::min<int32_t>(pages, (int32_t)(min_len / kPageTokens));
+      };
+      // A family larger than one tile is split into ceil(m / per_group)
+      // subgroups of near-equal size (7 at 6 per tile: 4 + 3), every one of
+      // them over the family's common pages, so that sibling items cover the
+      // same runs and can be scheduled together.
+      const size_t nm = mem.size(), n_sub = (nm + per_group - 1) / per_group;
+      const int32_t fam_pages = n_sub > 1 ? common_pages(0, nm) : 0;
+      for (size_t sg = 0; sg < n_sub; ++sg) {
+        const size_t b0 = sg * nm / n_sub, b1 = (sg + 1) * nm / n_sub;
+        if (n_sub == 1 && b1 - b0 < 2) continue;  // a lone sequence reads its pages as its own
+        const int32_t pages = n_sub > 1 ? fam_pages : common_pages(b0, b1);
         if (pages < 1) continue;
         Group g;
         g.members.assign(mem.begin() + b0, mem.begin() + b1);
         g.pages = pages;
+        g.family = f;
+        g.split = n_sub > 1;
         for (int i : g.members) shared[i] = pages;
         groups.push_back(std::move(g));
       }
@@ -658,6 +671,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   if (st != ST_OK) return st;
 
   std::vector<AttnItem> items;
+  std::vector<int32_t> item_family;  // fork family of a subgroup's item, for scheduling siblings together
   std::vector<int32_t> members;
   std::vector<int32_t> n_splits(n_br, 0);
   double bytes = 0, flops = 0;
@@ -670,7 +684,8 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
       int32_t b, n;
       split_even(g.pages, k, cidx, &b, &n);
       items.push_back(AttnItem{slots[g.members[0]], b, n, n * kPageTokens, mbase,
-                               (int32_t)g.members.size(), cidx, 0});
+                               (int32_t)g.members.size(), cidx, g.split ? 1 : 0});
+      item_family.push_back(g.family);
       bytes += n * page_bytes;
       flops += 4.0 * g.members.size() * G * n * kPageTokens * c.head_dim;
     }
@@ -687,14 +702,28 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
       split_even(own_pages[i], k, cidx, &b, &n);
       const int32_t tok = std::min<int32_t>(n * kPageTokens, own_tokens[i] - b * kPageTokens);
       items.push_back(AttnItem{slots[i], shared[i] + b, n, tok, mbase, 1, n_splits[i] + cidx, 0});
+      item_family.push_back(-1);
       bytes += n * page_bytes;
       flops += 4.0 * G * tok * c.head_dim;
     }
     n_splits[i] += k;
   }
-  // longest runs first so the short ones fill the tail
-  std::stable_sort(items.begin(), items.end(),
-                   [](const AttnItem& a, const AttnItem& b) { return a.n_pages > b.n_pages; });
+  // longest runs first so the short ones fill the tail; the items of a split
+  // group's subgroups over the same pages next to each other (same length,
+  // family and first page), so that the second read hits L2
+  {
+    std::vector<int> order(items.size());
+    for (size_t i = 0; i < order.size(); ++i) order[i] = (int)i;
+    auto key = [&](int i) {
+      const AttnItem& a = items[i];
+      return std::make_tuple(-a.n_pages, a.reread ? 0 : 1, a.reread ? item_family[i] : 0,
+                             a.reread ? a.page_begin : 0);
+    };
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return key(a) < key(b); });
+    std::vector<AttnItem> sorted(items.size());
+    for (size_t i = 0; i < order.size(); ++i) sorted[i] = items[order[i]];
+    items.swap(sorted);
+  }
   bytes *= (double)c.n_kv_heads * c.n_layers;
   flops *= (double)c.n_kv_heads * c.n_layers;
   const double q_bytes = (double)c.n_layers * n_br * c.n_q_heads * c.head_dim * 2;

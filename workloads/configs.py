@@ -72,16 +72,25 @@ def _batched():
         limits=dict(max_seqs=96, max_decode_branches=80, max_splits=16, max_pages=2304))
 
 
-def _long():
+def _long(n_aux=4):
     import numpy as np
     rng = np.random.default_rng(3)
-    S = tuple(tuple(int(x) for x in rng.integers(0, 2048, size=5, endpoint=True)) for _ in range(4))
+    S = tuple(tuple(int(x) for x in rng.integers(0, 2048, size=n_aux + 1, endpoint=True)) for _ in range(4))
     # room for every suffix plus 256 decode steps per branch
     pages = sum(131072 // 16 + sum((s + 256 + 15) // 16 + 1 for s in row) for row in S)
+    name = "long_trajectory_agent" if n_aux == 4 else f"long_trajectory_agent_{n_aux + 1}_branches"
     return Workload(
-        name="long_trajectory_agent", n_layers=32, n_q_heads=64, n_kv_heads=8, head_dim=128,
+        name=name, n_layers=32, n_q_heads=64, n_kv_heads=8, head_dim=128, n_aux=n_aux,
         n_blocks=pages + 64, seed=3, n_tasks=4, prefix=(131072,) * 4, suffix=S, steps=1,
-        limits=dict(max_seqs=24, max_decode_branches=20, max_splits=32, max_pages=8192 + 160))
+        limits=dict(max_seqs=4 * (n_aux + 1) + 4, max_decode_branches=4 * (n_aux + 1), max_splits=32,
+                    max_pages=8192 + 160))
+
+
+def long_with_branches(n_aux: int) -> Workload:
+    """The long-trajectory workload with n_aux auxiliary branches per group
+    (Section 3.2 lets the branch count vary): 1 + n_aux branches x 8 query
+    heads per KV head are stacked on each shared page."""
+    return _long(n_aux)
 
 
 def _cycle():
