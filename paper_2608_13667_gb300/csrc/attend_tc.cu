@@ -7,29 +7,36 @@
 // pages of one KV head of one layer and stacks every query row that reads
 // it -- for a shared prefix all branches of the fork group x the G query
 // heads of the KV head (<= 48 rows) -- so each prefix page crosses HBM once
-// per group.  A group with more than 48 stacked rows (more than 48 / G
-// branches; Section 3.2 lets the branch count vary) is split into subgroups
-// whose items over the same pages run next to each other, so the second
-// read of a page comes from L2.
+// per group.
+//
+// Two tile shapes (Section 3.2 lets the branch count vary, so the stacked
+// row count n_b G does):
+//   narrow  M = 64, up to 48 rows (the paper's 1 + 4 branches at G <= 9);
+//           P goes to shared memory over the stage's consumed K slot
+//   wide    M = 128, up to 128 rows; P stays in TMEM over its own scores and
+//           P V reads it from there (no P in shared memory, so two CTAs still
+//           fit an SM).
+// A group beyond 128 rows is split into subgroups whose items over the same
+// pages run next to each other, so the second read of a page comes from L2.
 //
 // CTA layout (192 threads, 2 CTAs per SM):
-//   warps 0..3  softmax (only ceil(rows/16) of them run).  The MMA is
-//               M = 64: row r sits in TMEM lane 32 (r / 16) + r % 16, and
-//               threads t and t + 16 of a warp share row t, each with half of
-//               the stage's keys and half of the O columns (16-lane TMEM
-//               loads with a column split).  A thread loads its half of its
-//               Q row into shared memory; per stage it reads its scores from
-//               TMEM, masks keys past the run, keeps a running max (combined
-//               with its partner by one shuffle) that is raised only when a
-//               score exceeds it by more than 2^8 (O in TMEM is then rescaled
-//               in place), and writes P = 2^(s - m) as two bf16 terms over the
-//               stage's consumed K slot.  At the end it normalises O out of
-//               TMEM: a split-KV partial with its log-sum-exp.
+//   warps 0..3  softmax (only those with rows run).  Narrow: row r sits in
+//               TMEM lane 32 (r / 16) + r % 16, and threads t and t + 16 of a
+//               warp share row t, each with half of the stage's keys and half
+//               of the O columns (16-lane TMEM loads with a column split).
+//               Wide: thread r owns row r = TMEM lane r.  A thread loads its
+//               part of its Q row into shared memory; per stage it reads its
+//               scores from TMEM, masks keys past the run, keeps a running max
+//               (narrow: combined with its partner by one shuffle) that is
+//               raised only when a score exceeds it by more than 2^8 (O in
+//               TMEM is then rescaled in place), and writes P = 2^(s - m) as
+//               two bf16 terms.  At the end it normalises O out of TMEM: a
+//               split-KV partial with its log-sum-exp.
 //   warp 4      loader: page ids from the block table (32 per read, one batch
 //               ahead), one 2 KiB TMA copy per (page, 64-wide half of D, K|V)
 //               into a ring of stages, per-stage mbarriers with byte counts.
-//   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M=64, N=64 keys)
-//               and O += P V (M=64, N=D) and commits them to mbarriers.  S is
+//   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M, N=64 keys)
+//               and O += P V (M, N=D) and commits them to mbarriers.  S is
 //               double-buffered in TMEM: S_{j+1} is issued before P_j V_j when
 //               its data has landed, so the softmax of stage j+1 overlaps the
 //               tensor work of stage j.
@@ -38,10 +45,12 @@
 // Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
 //   Q  [D/64][rows][64]       K-major A (SBO 1024)
 //   K  [D/64][keys][64]       K-major B (SBO 1024)
-//   P  [rows][keys]           K-major A (SBO 1024), written over K: two bf16
-//                             terms P_hi, P_lo, one after the other
+//   P  [rows][keys]           narrow: K-major A (SBO 1024), written over K: two
+//                             bf16 terms P_hi, P_lo, one after the other
+//                             wide: in TMEM, the 16 score columns of keys
+//                             [16 k, 16 k + 16) holding P_hi and P_lo of them
 //   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
-// The MMA computes 64 rows and only the first <= 48 Q and P rows are
+// The narrow MMA computes 64 rows and only the first <= 48 Q and P rows are
 // written; rows past them read whatever follows in shared memory and only
 // produce accumulator rows that nobody reads (each output row depends on its
 // own A row only).  V rows of keys that are not valid (past the run,
@@ -66,24 +75,25 @@ constexpr int kMaxDevices = 64;
 
 constexpr int cmax(int a, int b) { return a > b ? a : b; }
 
-template <int D>
+template <int D, bool kWide>
 struct TcCfg {
   static constexpr int kHalves = D / 64;
   static constexpr int kKeys = 64;                     // keys per stage
   static constexpr int kPagesPerStage = kKeys / kPageTokens;
-  static constexpr int kStages = 3;
+  static constexpr int kStages = kWide ? 2 : 3;
   // MMA M = 64 for <= 48 stacked rows: accumulator rows sit in TMEM lanes
-  // 0..15 of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16)
-  static constexpr int kM = 64;
+  // 0..15 of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
+  // M = 128 for up to 128 rows (row r at lane r)
+  static constexpr int kM = kWide ? 128 : 64;
   static constexpr int kRowsPerWarp = kM / 4;
-  static constexpr int kQRows = 48;                    // Q/P rows stored
+  static constexpr int kQRows = kWide ? 128 : 48;      // Q rows stored
   static constexpr int kQHalfBytes = kQRows * 128;
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kKVHalfBytes = kKeys * 128;
   // P as two bf16 terms (P = P_hi + P_lo, two MMAs against the same V): the
   // rounding of a single bf16 P does not average out when a row sees few
-  // keys or its weights are peaked
-  static constexpr int kPTermBytes = kQRows * 128;                // one term, kQRows rows
+  // keys or its weights are peaked.  Narrow: both terms over the K slot.
+  static constexpr int kPTermBytes = kWide ? 0 : kQRows * 128;    // one term, kQRows rows
   static constexpr int kPloOffset = kPTermBytes;                  // P_lo after P_hi in the K slot
   static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, 2 * kPTermBytes);
   static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
@@ -91,16 +101,16 @@ struct TcCfg {
   static constexpr int kRingBytes = kStages * kStageBytes;
   // the MMA reads kM rows of each P term from the last K slot: keep that
   // inside the allocation
-  static constexpr int kOverread = cmax(0, kPloOffset + kM * 128 - kStageBytes);
+  static constexpr int kOverread = kWide ? 0 : cmax(0, kPloOffset + kM * 128 - kStageBytes);
   static constexpr int kBarOffset = kQBytes + kRingBytes + kOverread;
   static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 };
 
-template <int D>
+template <int D, bool kWide>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
-  using C = TcCfg<D>;
+  using C = TcCfg<D, kWide>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
@@ -124,7 +134,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 
   // ---- what this CTA reads and for whom ------------------------------------------
   const int32_t* members = p.members ? p.members : inl.members;
-  const AttnItem item = p.items ? p.items[blockIdx.x] : inl.items[blockIdx.x];
+  const int item_idx = p.item_base + blockIdx.x;
+  const AttnItem item = p.items ? p.items[item_idx] : inl.items[item_idx];
   const int slot = item.slot;
   const int page_begin = item.page_begin;
   const int n_pages = item.n_pages;
@@ -163,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     // a page is streamed once, unless a sibling item (the group's other
     // subgroup, scheduled next to this one) reads it too: then keep it in L2
-    const uint64_t policy = item.reread ? l2_policy_evict_normal() : l2_policy_evict_first();
+    const uint64_t policy = (item.flags & kItemReread) ? l2_policy_evict_normal() : l2_policy_evict_first();
     const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
@@ -268,15 +279,26 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int s = j % C::kStages;
         const uint32_t k_addr = smem_addr(ring + s * C::kStageBytes);
         const uint32_t v_addr = k_addr + C::kKSlotBytes;
+        if constexpr (kWide) {
+          // P_hi, P_lo of keys [16 ks, 16 ks + 16) in the 16 TMEM columns of their scores
+          const uint32_t p_tm = tmem + kTmemS + (j & 1) * C::kKeys;
 #pragma unroll
-        for (int ks = 0; ks < C::kKeys / 16; ++ks)
-          tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + ks * 32, 16, 1024),
-                      tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
-                      (j > 0 || ks > 0) ? 1u : 0u);
+          for (int ks = 0; ks < C::kKeys / 16; ++ks) {
+            const uint64_t vd = tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024);
+            tc_mma_bf16_tmem_a(tmem + kTmemO, p_tm + ks * 16, vd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
+            tc_mma_bf16_tmem_a(tmem + kTmemO, p_tm + ks * 16 + 8, vd, idesc_o, 1u);
+          }
+        } else {
 #pragma unroll
-        for (int ks = 0; ks < C::kKeys / 16; ++ks)
-          tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
-                      tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
+          for (int ks = 0; ks < C::kKeys / 16; ++ks)
+            tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + ks * 32, 16, 1024),
+                        tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
+                        (j > 0 || ks > 0) ? 1u : 0u);
+#pragma unroll
+          for (int ks = 0; ks < C::kKeys / 16; ++ks)
+            tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
+                        tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
+        }
         tc_commit(&empty[s]);
         tc_commit(o_ready);
         if (jn < n_tiles && !early && !issue_s(jn)) {
@@ -296,13 +318,15 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (warp >= n_sw) return;
 
   // ---- softmax warps ---------------------------------------------------------------
-  // Threads t and t + 16 of a warp share row t: half of the stage's keys and
-  // half of the O columns each, the row max and sum combined with one shuffle.
-  constexpr int kKpt = C::kKeys / 2;  // keys per thread per stage
-  constexpr int kOpt = D / 2;         // O columns per thread
-  const int tid = threadIdx.x;        // 0 .. n_swt-1, for cooperative loops
-  const int half = lane >> 4;
-  const int r = warp * 16 + (lane & 15);  // this thread's row
+  // Narrow: threads t and t + 16 of a warp share row t, half of the stage's
+  // keys and half of the O columns each, the row max and sum combined with
+  // one shuffle.  Wide: one thread per row.
+  constexpr bool kPair = !kWide;
+  constexpr int kKpt = C::kKeys / (kPair ? 2 : 1);  // keys per thread per stage
+  constexpr int kOpt = D / (kPair ? 2 : 1);         // O columns per thread
+  const int tid = threadIdx.x;                      // 0 .. n_swt-1, for cooperative loops
+  const int half = kPair ? (lane >> 4) : 0;
+  const int r = kPair ? warp * 16 + (lane & 15) : threadIdx.x;  // this thread's row
   const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
   const bool valid = r < n_rows;
   int qrow = 0, head = 0;
@@ -312,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   if (r < C::kQRows) {
     const uint4* src = reinterpret_cast<const uint4*>(p.q + (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * D);
-    constexpr int kChunks = D / 16;  // 16-byte chunks of the half row this thread writes
+    constexpr int kChunks = D / 8 / (kPair ? 2 : 1);  // 16-byte chunks of the row this thread writes
 #pragma unroll
     for (int cc = 0; cc < kChunks; ++cc) {
       const int c = half * kChunks + cc;
@@ -324,8 +348,14 @@ __global__ void __launch_bounds__(kThreads, 2)
   mbar_arrive(q_ready);
 
   // this thread's 32-column pieces of its O row: [o_col(k), o_col(k) + 32)
-  auto o_load = [&](int k, float* o) { tmem_ld16x2_32<D / 2>(t_lane + kTmemO + k * 32, o); };
-  auto o_store = [&](int k, const float* o) { tmem_st16x2_32<D / 2>(t_lane + kTmemO + k * 32, o); };
+  auto o_load = [&](int k, float* o) {
+    if constexpr (kPair) tmem_ld16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
+    else tmem_ld32(t_lane + kTmemO + k * 32, o);
+  };
+  auto o_store = [&](int k, const float* o) {
+    if constexpr (kPair) tmem_st16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
+    else tmem_st32(t_lane + kTmemO + k * 32, o);
+  };
   auto o_col = [&](int k) { return half * (D / 2) + k * 32; };
 
   const float sl2 = p.scale_log2;
@@ -342,7 +372,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     // domain, x = s * sl2
     float sc[kKpt];
     static_assert(C::kKeys == 64, "64 keys per stage");
-    tmem_ld16x2_32<32>(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
+    if constexpr (kPair) tmem_ld16x2_32<32>(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
+    else tmem_ld64(t_lane + kTmemS + (j & 1) * C::kKeys, sc);
     const int key0 = j * C::kKeys;
     const int kbase = half * kKpt;  // this thread's first key within the stage
     const int np = min(C::kPagesPerStage, n_pages - j * C::kPagesPerStage);
@@ -360,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int c = 8; c < kKpt; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sc[c]);
     float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                      fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+    if constexpr (kPair) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
     const float m_new = fmaxf(m_used, mx * sl2);  // sl2 > 0: max commutes with the scale
     const bool need = valid && m_new > m_used + kRescaleThreshold;
     if (__any_sync(0xffffffffu, need)) {
@@ -385,8 +416,30 @@ __global__ void __launch_bounds__(kThreads, 2)
       l *= alpha;
       if (need) m_used = m_new;
     }
-    uint8_t* kslot = ring + s * C::kStageBytes;  // S_j has been consumed: P_j goes over K_j
-    if (valid) {
+    uint8_t* kslot = ring + s * C::kStageBytes;  // narrow: S_j has been consumed, P_j goes over K_j
+    if constexpr (kWide) {
+      // P_hi, P_lo of keys [16 k, 16 k + 16) over the 16 TMEM columns of their
+      // scores (all read above).  The store is warp-wide: rows past the
+      // item's take 2^-inf = 0.
+      const uint32_t p_tm = t_lane + kTmemS + (j & 1) * C::kKeys;
+      const float mo = valid ? m_used : INFINITY;
+      float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int kq = 0; kq < C::kKeys / 16; ++kq) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int c = 0; c < 16; c += 2) {
+          const float a = ex2(fmaf(sc[kq * 16 + c], sl2, -mo)), b = ex2(fmaf(sc[kq * 16 + c + 1], sl2, -mo));
+          rs[(c >> 1) & 7] += a + b;
+          const uint32_t hi = pack_bf16(a, b);
+          pk[c / 2] = hi;
+          pk[8 + c / 2] = pack_bf16(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
+        }
+        tmem_st16u_nowait(p_tm + kq * 16, pk);
+      }
+      tmem_wait_st();
+      l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
+    } else if (valid) {
       uint32_t pk[kKpt / 2];
       uint32_t pl[kKpt / 2];
       float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -430,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0));
   tc_fence_after_sync();
   if (ok) {
-    l += __shfl_xor_sync(0xffffffffu, l, 16);  // the row's full sum
+    if constexpr (kPair) l += __shfl_xor_sync(0xffffffffu, l, 16);  // the row's full sum
     const float inv = 1.f / l;
     float* dst = nullptr;
     float* dst_lse = nullptr;
@@ -458,10 +511,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   named_barrier_sync(1, n_swt + 32);
 }
 
-template <int D>
+template <int D, bool kWide>
 cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
                         const InlineDecodePlan& inl, int n_ctas, cudaStream_t s) {
-  using C = TcCfg<D>;
+  using C = TcCfg<D, kWide>;
   // the shared-memory opt-in is a per-device function attribute
   static bool configured[kMaxDevices] = {};
   int dev = 0;
@@ -469,23 +522,24 @@ cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const Attn
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    e = cudaFuncSetAttribute(attend_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    e = cudaFuncSetAttribute(attend_tc_kernel<D, kWide>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  attend_tc_kernel<D><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
+  attend_tc_kernel<D, kWide><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
   return cudaGetLastError();
 }
 
 template <int D>
 int decode_ctas_per_sm_t() {
-  using C = TcCfg<D>;
-  if (cudaFuncSetAttribute(attend_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
-      cudaSuccess)
+  using C = TcCfg<D, false>;
+  if (cudaFuncSetAttribute(attend_tc_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           C::kSmemBytes) != cudaSuccess)
     return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D>, kThreads, C::kSmemBytes) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, false>, kThreads, C::kSmemBytes) !=
       cudaSuccess)
     return 0;
   return n < 2 ? n : 2;  // two CTAs' TMEM (2 x 256 columns) fill an SM
@@ -494,12 +548,14 @@ int decode_ctas_per_sm_t() {
 }  // namespace
 
 cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
-                             const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s) {
+                             const InlineDecodePlan* inl, int n_items, int D, bool wide, cudaStream_t s) {
   static const InlineDecodePlan kNone{};
   const InlineDecodePlan& ip = inl ? *inl : kNone;
   if (n_items <= 0) return cudaSuccess;
-  if (D == 128) return launch_tc_t<128>(km, vm, p, ip, n_items, s);
-  if (D == 64) return launch_tc_t<64>(km, vm, p, ip, n_items, s);
+  if (D == 128)
+    return wide ? launch_tc_t<128, true>(km, vm, p, ip, n_items, s) : launch_tc_t<128, false>(km, vm, p, ip, n_items, s);
+  if (D == 64)
+    return wide ? launch_tc_t<64, true>(km, vm, p, ip, n_items, s) : launch_tc_t<64, false>(km, vm, p, ip, n_items, s);
   return cudaErrorInvalidValue;
 }
 

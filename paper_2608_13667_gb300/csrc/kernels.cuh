@@ -61,8 +61,12 @@ struct AttnItem {
   int32_t member_base; // index of the first member in the members array
   int32_t n_members;
   int32_t split;       // partial slot this item writes
-  int32_t reread;      // 1: a sibling item (another subgroup of the fork group) reads the same pages
+  int32_t flags;       // kItemReread | kItemWide
 };
+// a sibling item (another subgroup of the fork group) reads the same pages
+constexpr int32_t kItemReread = 1;
+// more than 48 stacked rows: the M = 128 tile
+constexpr int32_t kItemWide = 2;
 
 struct AttnParams {
   const __nv_bfloat16* q;  // [L][n_rows_q][Hq][D]
@@ -78,6 +82,7 @@ struct AttnParams {
   int32_t Hq, Hkv, G, L, max_pages, max_splits;
   int32_t slot, L0, T;     // merge only: main's slot, length before the append, thought rows
   int32_t hold_loads;      // test hook (ST_FLAG_HOLD_LOADS): the loader issues nothing
+  int32_t item_base;       // decode: CTA x reads item item_base + x
 };
 
 struct CombineParams {
@@ -111,9 +116,10 @@ cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int3
                                 int n_runs, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, int D, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, int D, cudaStream_t s);
-// Decode partials on tcgen05 (one CTA per item x KV head x layer).
+// Decode partials on tcgen05 (one CTA per item x KV head x layer; items from
+// p.item_base on; wide: the M = 128 tile, for items flagged kItemWide).
 cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
-                             const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s);
+                             const InlineDecodePlan* inl, int n_items, int D, bool wide, cudaStream_t s);
 // Causal merge prefill on tcgen05 (p.slot, p.L0, p.T, p.q -> p.out_o, p.out_lse),
 // two 128-row query tiles per CTA sharing K/V (merge_tc.cu).
 cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int D,

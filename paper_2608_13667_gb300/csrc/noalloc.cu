@@ -235,7 +235,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   ap.L = c.n_layers;
   ap.max_pages = table_stride;
   ap.max_splits = kSplitStride;
-  if (launch_decode_tc(kmap, vmap, ap, nullptr, n_items, c.head_dim, s) != cudaSuccess) return ST_ERR_CUDA;
+  if (launch_decode_tc(kmap, vmap, ap, nullptr, n_items, c.head_dim, false, s) != cudaSuccess) return ST_ERR_CUDA;
   CombineParams cp{};
   cp.part_o = ap.out_o;
   cp.part_lse = ap.out_lse;

@@ -30,7 +30,8 @@ namespace {
 
 constexpr int kStageSlots = 8;
 constexpr size_t kStageSlotBytes = 2u << 20;  // 2 MiB per plan
-constexpr int kMaxAttnRows = 48;              // stacked query rows per CTA
+constexpr int kMaxAttnRows = 48;              // stacked query rows of the narrow decode tile
+constexpr int kMaxWideRows = 128;             // ... and of the wide one
 
 enum KernelId { kKTable = 0, kKAppend, kKDecode, kKCombine, kKMerge, kNumKernels };
 const char* const kKernelNames[kNumKernels] = {"table_update", "append_kv", "decode_partial",
@@ -603,7 +604,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
 
   // ---- group by fork family, find the shared full pages --------------------
   std::vector<int32_t> shared(n_br, 0);   // pages of branch i read through its group
-  struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split; };
+  struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split, wide; };
   std::vector<Group> groups;
   {
     std::map<int32_t, std::vector<int>> fam;
@@ -613,9 +614,12 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
       if (!fam.count(f)) order.push_back(f);
       fam[f].push_back(i);
     }
-    const int per_group = std::max(1, kMaxAttnRows / G);
     for (int32_t f : order) {
       const std::vector<int>& mem = fam[f];
+      // one narrow tile (<= 48 stacked rows), else one wide tile (<= 128), else
+      // wide subgroups
+      const bool wide = (int)mem.size() * G > kMaxAttnRows;
+      const int per_group = std::max(1, (wide ? kMaxWideRows : kMaxAttnRows) / G);
       // full pages held by every member of mem[b0, b1)
       auto common_pages = [&](size_t b0, size_t b1) {
         const SeqSlot& lead = bp.slot(slots[mem[b0]]);
@@ -644,6 +648,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
         g.pages = pages;
         g.family = f;
         g.split = n_sub > 1;
+        g.wide = wide;
         for (int i : g.members) shared[i] = pages;
         groups.push_back(std::move(g));
       }
@@ -683,8 +688,8 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     for (int32_t cidx = 0; cidx < k; ++cidx) {
       int32_t b, n;
       split_even(g.pages, k, cidx, &b, &n);
-      items.push_back(AttnItem{slots[g.members[0]], b, n, n * kPageTokens, mbase,
-                               (int32_t)g.members.size(), cidx, g.split ? 1 : 0});
+      items.push_back(AttnItem{slots[g.members[0]], b, n, n * kPageTokens, mbase, (int32_t)g.members.size(),
+                               cidx, (g.split ? kItemReread : 0) | (g.wide ? kItemWide : 0)});
       item_family.push_back(g.family);
       bytes += n * page_bytes;
       flops += 4.0 * g.members.size() * G * n * kPageTokens * c.head_dim;
@@ -708,16 +713,18 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     }
     n_splits[i] += k;
   }
-  // longest runs first so the short ones fill the tail; the items of a split
-  // group's subgroups over the same pages next to each other (same length,
-  // family and first page), so that the second read hits L2
+  // narrow items, then wide ones (two launches); within each, longest runs
+  // first so the short ones fill the tail, and the items of a split group's
+  // subgroups over the same pages next to each other (same length, family and
+  // first page), so that the second read hits L2
   {
     std::vector<int> order(items.size());
     for (size_t i = 0; i < order.size(); ++i) order[i] = (int)i;
     auto key = [&](int i) {
       const AttnItem& a = items[i];
-      return std::make_tuple(-a.n_pages, a.reread ? 0 : 1, a.reread ? item_family[i] : 0,
-                             a.reread ? a.page_begin : 0);
+      const bool rr = (a.flags & kItemReread) != 0;
+      return std::make_tuple((a.flags & kItemWide) ? 1 : 0, -a.n_pages, rr ? 0 : 1, rr ? item_family[i] : 0,
+                             rr ? a.page_begin : 0);
     };
     std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return key(a) < key(b); });
     std::vector<AttnItem> sorted(items.size());
@@ -779,8 +786,15 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.max_splits = c.max_splits;
   ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
   const int n_items = (int)items.size();
+  int n_narrow = 0;
+  while (n_narrow < n_items && !(items[n_narrow].flags & kItemWide)) ++n_narrow;
   st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
-    return launch_decode_tc(P->kmap, P->vmap, ap, inline_plan ? &inl : nullptr, n_items, c.head_dim, s);
+    const InlineDecodePlan* ip = inline_plan ? &inl : nullptr;
+    cudaError_t e = launch_decode_tc(P->kmap, P->vmap, ap, ip, n_narrow, c.head_dim, false, s);
+    if (e != cudaSuccess || n_narrow == n_items) return e;
+    AttnParams aw = ap;
+    aw.item_base = n_narrow;
+    return launch_decode_tc(P->kmap, P->vmap, aw, ip, n_items - n_narrow, c.head_dim, true, s);
   });
   if (st != ST_OK) return st;
 
