@@ -162,12 +162,12 @@ def _small(D, Hq, Hkv, n_blocks=512, L=2, seed=11, scale=1.0):
     (128, 32, 8, 1, 1000, (5, 0)),
     (128, 8, 8, 7, 777, (1, 2, 3, 0, 16, 17, 31, 100)),      # G = 1, eight branches
     (128, 64, 8, 4, 300, (0, 1, 15, 16, 17)),                # G = 8, 40 stacked rows
-    (128, 64, 8, 8, 4100, (3,) * 9),                         # 9 x 8 = 72 rows: subgroups of 6 and 3
-    (128, 16, 1, 3, 2000, (0, 9, 0, 40)),                    # G = 16: subgroups of 3 (48 rows) and 1
-    (64, 48, 4, 7, 900, (2,) * 8),                           # G = 12, 96 rows: two full subgroups, D 64
-    (128, 32, 1, 3, 1500, (0, 5, 9, 33)),                    # G = 32: one branch per subgroup
-    (128, 48, 1, 4, 700, (1, 2, 3, 4, 5)),                   # G = 48: one branch per subgroup
-    (64, 20, 2, 5, 3333, (0, 7, 16, 31, 64, 65)),            # G = 10, 60 rows: subgroups of 4 and 2, D 64
+    (128, 64, 8, 8, 4100, (3,) * 9),                         # 9 x 8 = 72 rows: one wide tile
+    (128, 16, 1, 3, 2000, (0, 9, 0, 40)),                    # G = 16, 64 rows: wide
+    (64, 48, 4, 7, 900, (2,) * 8),                           # G = 12, 96 rows: wide, D 64
+    (128, 32, 1, 3, 1500, (0, 5, 9, 33)),                    # G = 32, 128 rows: a full wide tile
+    (128, 48, 1, 4, 700, (1, 2, 3, 4, 5)),                   # G = 48, 240 rows: wide subgroups 1 + 2 + 2
+    (64, 20, 2, 5, 3333, (0, 7, 16, 31, 64, 65)),            # G = 10, 60 rows: wide, D 64
     (128, 32, 1, 1, 100, (0, 0)),                            # G = 32, no suffixes
     (64, 4, 1, 0, 50, (0,)),                                 # a lone main thread
     (64, 12, 3, 2, 16, (0, 1, 2)),                           # one-page prefix
