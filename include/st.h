@@ -164,6 +164,25 @@ ST_API st_status st_decode_attn(st_pool* pool, const st_seq* br, int n_br, const
 ST_API st_status st_merge(st_pool* pool, st_seq main, int n_tok, const void* q, const void* k,
                           const void* v, float* o, float* lse, void* stream);
 
+/* Batched prefill across sequences (Section 3.1: the observation O_t is
+ * appended to each agent's history, and Section 3.5: the harvested thoughts
+ * after it; several agents' rows arrive together when many are served at
+ * once).  For each i in order, n_tok[i] rows are appended to seqs[i] (same
+ * rules as st_append_kv; the pages are taken as if the sequences were
+ * appended one after another) and run through the causal prefill of
+ * st_merge: row r of sequence i attends over its rows [0, L0_i + r], L0_i =
+ * its length before the call.  One launch covers every sequence.
+ * n_tok:  host int32 [n_seq], each >= 0 (0: the sequence is left unchanged)
+ * rows are packed in sequence order, R = sum of n_tok:
+ * q: bf16 [n_layers][R][n_q_heads][head_dim];
+ * k, v: bf16 [n_layers][R][n_kv_heads][head_dim];
+ * o: fp32 [n_layers][R][n_q_heads][head_dim]; lse: fp32 [n_layers][R][n_q_heads].
+ * A sequence may appear once.  All or nothing on ST_ERR_OOM.  R = 0 is a
+ * no-op.  On a metadata-only pool all five pointers must be NULL. */
+ST_API st_status st_prefill_batch(st_pool* pool, const st_seq* seqs, int n_seq, const int32_t* n_tok,
+                                  const void* q, const void* k, const void* v, float* o, float* lse,
+                                  void* stream);
+
 /* Thought harvest (Section 3.5): when the observation arrives, each branch's
  * generated token stream is cut at its last closed </thought>.  Completed
  * atoms (an open-tag token through the next close-tag token, tags included)

@@ -155,17 +155,25 @@ class RefPool:
         ``labels[i][t]`` is stored as the content of row t of sequence i when
         content tracking is on.
         """
+        return self.prefill_batch(seq_ids, [n_tok] * len(seq_ids), labels)
+
+    def prefill_batch(self, seq_ids, counts, labels=None):
+        """Append counts[i] rows to sequence seq_ids[i], the sequences taken in
+        order: the bookkeeping of a batched prefill, in which several agents'
+        observation (Section 3.1) and thought (Section 3.5) rows arrive
+        together.  All or nothing."""
         assert len(set(seq_ids)) == len(seq_ids), "a sequence may appear once per call"
+        assert len(counts) == len(seq_ids) and all(n >= 0 for n in counts)
         seqs = [self.seqs[i] for i in seq_ids]
         assert all(s.alive for s in seqs)
         # all-or-nothing: the whole call's page need is checked first
-        if sum(self._pages_needed(s, n_tok) for s in seqs) > len(self.free):
+        if sum(self._pages_needed(s, n) for s, n in zip(seqs, counts)) > len(self.free):
             raise OutOfBlocks()
         events = []
         p = self.page
         for idx, i in enumerate(seq_ids):
             s = self.seqs[i]
-            for t in range(n_tok):
+            for t in range(counts[idx]):
                 off = s.length % p
                 if off == 0:
                     s.table.append(self._pop())

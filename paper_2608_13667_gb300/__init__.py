@@ -78,6 +78,7 @@ def lib():
         "st_append_kv": (I, [P, i64p, I, I, VP, VP, VP]),
         "st_decode_attn": (I, [P, i64p, I, VP, VP, VP, VP]),
         "st_merge": (I, [P, I64, I, VP, VP, VP, VP, VP, VP]),
+        "st_prefill_batch": (I, [P, i64p, I, i32p, VP, VP, VP, VP, VP, VP]),
         "st_release": (I, [P, I64]),
         "st_block_table": (I, [P, I64, i32p, I, ctypes.POINTER(I), ctypes.POINTER(I)]),
         "st_refcounts": (I, [P, i32p, I64]),
@@ -252,6 +253,36 @@ class Pool:
         self._check(lib().st_merge(self._h, int(main), T, qp, kp, vp, op, lp, self._stream(stream)), "st_merge")
         return o, lse
 
+    def prefill_batch(self, seqs, n_tok, q, k, v, o=None, lse=None, stream=None):
+        """n_tok[i] rows appended to seqs[i] and prefilled causally, all in one
+        launch.  Rows packed in sequence order (R = sum(n_tok)):
+        q: bf16 [L][R][Hq][D]; k, v: bf16 [L][R][Hkv][D] -> (o [L][R][Hq][D], lse [L][R][Hq]).
+        On a metadata-only pool pass q = k = v = None."""
+        c = self.cfg
+        arr, n = _seq_array(seqs)
+        counts = [int(x) for x in n_tok]
+        if len(counts) != n:
+            raise ValueError("n_tok needs one count per sequence")
+        cnt = (ctypes.c_int32 * max(1, n))(*counts)
+        if self.device is None:
+            self._check(lib().st_prefill_batch(self._h, arr, n, cnt, None, None, None, None, None, None),
+                        "st_prefill_batch")
+            return None, None
+        import torch
+        R = sum(counts)
+        qp = self._dev(q, torch.bfloat16, (c.n_layers, R, c.n_q_heads, c.head_dim), "q")
+        kp = self._dev(k, torch.bfloat16, (c.n_layers, R, c.n_kv_heads, c.head_dim), "k")
+        vp = self._dev(v, torch.bfloat16, (c.n_layers, R, c.n_kv_heads, c.head_dim), "v")
+        if o is None:
+            o = torch.empty((c.n_layers, R, c.n_q_heads, c.head_dim), dtype=torch.float32, device=self.device)
+        if lse is None:
+            lse = torch.empty((c.n_layers, R, c.n_q_heads), dtype=torch.float32, device=self.device)
+        op = self._dev(o, torch.float32, (c.n_layers, R, c.n_q_heads, c.head_dim), "o")
+        lp = self._dev(lse, torch.float32, (c.n_layers, R, c.n_q_heads), "lse")
+        self._check(lib().st_prefill_batch(self._h, arr, n, cnt, qp, kp, vp, op, lp, self._stream(stream)),
+                    "st_prefill_batch")
+        return o, lse
+
     def release(self, seq):
         self._check(lib().st_release(self._h, int(seq)), "st_release")
 
@@ -318,6 +349,10 @@ def st_decode_attn(pool, branches, q, o=None, lse=None, stream=None):
 
 def st_merge(pool, main, q, k, v, o=None, lse=None, stream=None):
     return pool.merge(main, q, k, v, o, lse, stream)
+
+
+def st_prefill_batch(pool, seqs, n_tok, q, k, v, o=None, lse=None, stream=None):
+    return pool.prefill_batch(seqs, n_tok, q, k, v, o, lse, stream)
 
 
 def st_release(pool, seq):

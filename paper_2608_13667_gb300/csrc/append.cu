@@ -22,7 +22,8 @@ __global__ void table_update_kernel(int32_t* __restrict__ table, const TableRun*
 
 // One thread moves 16 bytes (8 bf16).  Index space: copy-on-write chunks
 // first (n_cow x L x Hkv x 16 rows x D/8, rows past the copy length idle),
-// then the appended rows in the input's own order [L][n_br][n_tok][Hkv][D/8].
+// then the appended rows in the input's own order [L][n_rows][Hkv][D/8];
+// row r belongs to the branch whose [row0, row0 + n) holds it.
 template <int D>
 __global__ void __launch_bounds__(256) append_kernel(const AppendParams p,
                                                      const __grid_constant__ InlineAppendPlan inl) {
@@ -30,7 +31,7 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p,
   const CowCopy* cows = p.cows ? p.cows : inl.cows;
   constexpr int kChunks = D / 8;
   const int64_t cow_total = (int64_t)p.n_cow * p.L * p.Hkv * kPageTokens * kChunks;
-  const int64_t app_total = (int64_t)p.L * p.n_br * p.n_tok * p.Hkv * kChunks;
+  const int64_t app_total = (int64_t)p.L * p.n_rows * p.Hkv * kChunks;
   const int64_t total = cow_total + app_total;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
@@ -56,11 +57,22 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p,
       int64_t x = j;
       const int c = (int)(x % kChunks); x /= kChunks;
       const int g = (int)(x % p.Hkv); x /= p.Hkv;
-      const int t = (int)(x % p.n_tok); x /= p.n_tok;
-      const int b = (int)(x % p.n_br); x /= p.n_br;
+      const int row = (int)(x % p.n_rows); x /= p.n_rows;
       const int l = (int)x;
+      int b;
+      if (p.ragged) {  // the last branch whose first row is <= row
+        int lo = 0, hi = p.n_br - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (branches[mid].row0 <= row) lo = mid;
+          else hi = mid - 1;
+        }
+        b = lo;
+      } else {
+        b = row / p.n_tok;
+      }
       const AppendBranch br = branches[b];
-      const int pos = br.start + t;
+      const int pos = br.start + (row - br.row0);
       const int32_t blk = p.table[(int64_t)br.slot * p.max_pages + pos / kPageTokens];
       if ((uint64_t)blk >= (uint64_t)p.n_blocks) {
         atomicCAS(p.status, 0, kDevBadIndex);
@@ -100,7 +112,7 @@ cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, in
   static const InlineAppendPlan kNone{};
   const InlineAppendPlan& ip = inl ? *inl : kNone;
   const int64_t total = (int64_t)p.n_cow * p.L * p.Hkv * kPageTokens * (D / 8) +
-                        (int64_t)p.L * p.n_br * p.n_tok * p.Hkv * (D / 8);
+                        (int64_t)p.L * p.n_rows * p.Hkv * (D / 8);
   if (total == 0) return cudaSuccess;
   const int grid = grid_for(total, 256);
   if (D == 128)

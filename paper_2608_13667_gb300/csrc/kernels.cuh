@@ -36,10 +36,12 @@ struct CowCopy {
 struct AppendBranch {
   int32_t slot;
   int32_t start;  // sequence length before this call
+  int32_t row0;   // first of this branch's rows in the call's input
+  int32_t n;      // rows appended to this branch
 };
 
 struct AppendParams {
-  const __nv_bfloat16* k;  // [L][n_br][n_tok][Hkv][D]
+  const __nv_bfloat16* k;  // [L][n_rows][Hkv][D]: branch b's rows are [row0, row0 + n)
   const __nv_bfloat16* v;
   __nv_bfloat16* k_pool;   // [L][n_blocks][Hkv][16][D]
   __nv_bfloat16* v_pool;
@@ -49,6 +51,8 @@ struct AppendParams {
   int32_t* status;
   int64_t n_blocks;
   int32_t n_cow, n_br, n_tok, L, Hkv, max_pages;
+  int32_t n_rows;          // n_br * n_tok, or the sum of the branches' n
+  int32_t ragged;          // 0: every branch takes n_tok rows (branch of row r is r / n_tok)
 };
 
 // One unit of decode work: a run of pages of one block table, read for a set
@@ -68,21 +72,33 @@ constexpr int32_t kItemReread = 1;
 // more than 48 stacked rows: the M = 128 tile
 constexpr int32_t kItemWide = 2;
 
+// One CTA of a batched merge / prefill: rows [row_base, row_base + 256) of
+// one sequence's stacked (new row, head) rows.
+struct MergeItem {
+  int32_t slot;
+  int32_t L0;      // the sequence's length before this call
+  int32_t T;       // rows appended to it
+  int32_t q_row0;  // its first row in the call's Q / O / LSE
+  int32_t row_base;
+  int32_t pad[3];
+};
+
 struct AttnParams {
   const __nv_bfloat16* q;  // [L][n_rows_q][Hq][D]
-  float* out_o;            // decode: partials [L][n_br][Hq][max_splits][D]; merge: [L][T][Hq][D]
-  float* out_lse;          // decode: [L][n_br][Hq][max_splits];              merge: [L][T][Hq]
+  float* out_o;            // decode: partials [L][n_br][Hq][max_splits][D]; merge: [L][n_rows_q][Hq][D]
+  float* out_lse;          // decode: [L][n_br][Hq][max_splits];              merge: [L][n_rows_q][Hq]
   const int32_t* table;
   const AttnItem* items;   // decode only
   const int32_t* members;  // decode only: branch index (in the call) of each member
   int32_t* status;
   int64_t n_blocks;
   float scale_log2;        // log2(e) / sqrt(D)
-  int32_t n_rows_q;        // decode: n_br; merge: T
+  int32_t n_rows_q;        // decode: n_br; merge: rows in Q (T, or all sequences' rows)
   int32_t Hq, Hkv, G, L, max_pages, max_splits;
   int32_t slot, L0, T;     // merge only: main's slot, length before the append, thought rows
   int32_t hold_loads;      // test hook (ST_FLAG_HOLD_LOADS): the loader issues nothing
   int32_t item_base;       // decode: CTA x reads item item_base + x
+  const MergeItem* mitems; // batched merge: CTA x takes mitems[x] (slot, L0, T above unused)
 };
 
 struct CombineParams {
@@ -120,10 +136,11 @@ cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, 
 // p.item_base on; wide: the M = 128 tile, for items flagged kItemWide).
 cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
                              const InlineDecodePlan* inl, int n_items, int D, bool wide, cudaStream_t s);
-// Causal merge prefill on tcgen05 (p.slot, p.L0, p.T, p.q -> p.out_o, p.out_lse),
-// two 128-row query tiles per CTA sharing K/V (merge_tc.cu).
-cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int D,
-                            cudaStream_t s);
+// Causal merge prefill on tcgen05, two 128-row query tiles per CTA sharing
+// K/V (merge_tc.cu): one sequence (p.slot, p.L0, p.T; p.mitems null) or a
+// batch of n_items work items (p.mitems), p.q -> p.out_o, p.out_lse.
+cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int n_items,
+                            int D, cudaStream_t s);
 // CTAs of the tcgen05 decode kernel resident per SM (0 on error).
 int decode_tc_ctas_per_sm(int D);
 

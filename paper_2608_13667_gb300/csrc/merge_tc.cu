@@ -123,11 +123,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int layer = blockIdx.z;
   const int G = p.G;
 
-  const int row_base = blockIdx.x * 2 * kTileRows;
-  const int n_rows = min(2 * kTileRows, p.T * G - row_base);
+  // one merge: its row tiles in blockIdx.x order; a batch: one work item per CTA
+  int slot = p.slot, L0 = p.L0, T = p.T, q_row0 = 0, row_base = blockIdx.x * 2 * kTileRows;
+  if (p.mitems) {
+    const MergeItem mi = p.mitems[blockIdx.x];
+    slot = mi.slot;
+    L0 = mi.L0;
+    T = mi.T;
+    q_row0 = mi.q_row0;
+    row_base = mi.row_base;
+  }
+  const int n_rows = min(2 * kTileRows, T * G - row_base);
   const int t_last = (row_base + n_rows - 1) / G;
-  const int n_pages = (p.L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
-  const int n_valid_keys = p.L0 + p.T;
+  const int n_pages = (L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
+  const int n_valid_keys = L0 + T;
   const int n_tiles = (n_pages + kPagesPerStage - 1) / kPagesPerStage;
 
   if (threadIdx.x == 0) {
@@ -166,7 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) prefetch_tensormap(map);
     // every CTA of one (layer, KV head) walks the same pages: keep them in L2
     const uint64_t policy = l2_policy_evict_last();
-    const int32_t* ids = p.table + (int64_t)p.slot * p.max_pages;
+    const int32_t* ids = p.table + (int64_t)slot * p.max_pages;
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
     int nxt = 32 + lane < n_pages ? ids[32 + lane] : 0;
@@ -318,10 +327,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     qrow = gr / G;
     head = kvh * G + gr % G;
   }
-  const int limit = valid ? p.L0 + qrow + 1 : n_valid_keys;
-  const int min_limit = p.L0 + tile_row0 / G + 1;  // the tile's first row sees the fewest keys
+  const int limit = valid ? L0 + qrow + 1 : n_valid_keys;
+  const int min_limit = L0 + tile_row0 / G + 1;  // the tile's first row sees the fewest keys
+  const int64_t io_row = (int64_t)layer * p.n_rows_q + q_row0 + qrow;  // this row in Q / O / LSE
   {
-    const uint4* src = reinterpret_cast<const uint4*>(p.q + (((int64_t)layer * p.n_rows_q + qrow) * p.Hq + head) * D);
+    const uint4* src = reinterpret_cast<const uint4*>(p.q + (io_row * p.Hq + head) * D);
     uint8_t* q_s = base + C::kQOff + t * C::kQTileBytes;
 #pragma unroll
     for (int c = 0; c < D / 8; ++c) {
@@ -447,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after_sync();
   if (ok) {
     const float inv = 1.f / l;
-    float* dst = valid ? p.out_o + (((int64_t)layer * p.T + qrow) * p.Hq + head) * D : nullptr;
+    float* dst = valid ? p.out_o + (io_row * p.Hq + head) * D : nullptr;
 #pragma unroll 1
     for (int k = 0; k < D / 32; ++k) {
       float o[32];
@@ -459,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               make_float4(o[i] * inv, o[i + 1] * inv, o[i + 2] * inv, o[i + 3] * inv);
       }
     }
-    if (valid) p.out_lse[((int64_t)layer * p.T + qrow) * p.Hq + head] = (m_used + log2f(l)) * kLn2;
+    if (valid) p.out_lse[io_row * p.Hq + head] = (m_used + log2f(l)) * kLn2;
   } else if (lane == 0) {
     atomicCAS(p.status, 0, kDevTimeout);
   }
@@ -468,7 +478,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int D>
-cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, cudaStream_t s) {
+cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_ctas,
+                          cudaStream_t s) {
   using C = PairCfg<D>;
   // the shared-memory opt-in is a per-device function attribute
   static bool configured[64] = {};
@@ -481,18 +492,20 @@ cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const At
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  dim3 grid((p.T * p.G + 2 * kTileRows - 1) / (2 * kTileRows), p.Hkv, p.L);
+  dim3 grid(n_ctas, p.Hkv, p.L);
   merge_pair_kernel<D><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int D,
-                            cudaStream_t s) {
-  if (p.T <= 0) return cudaSuccess;
-  if (D == 128) return launch_pair_t<128>(km, vm, p, s);
-  if (D == 64) return launch_pair_t<64>(km, vm, p, s);
+cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_items,
+                            int D, cudaStream_t s) {
+  // one merge: ceil(T G / 256) row tiles; a batch: its work items
+  const int n_ctas = p.mitems ? n_items : (p.T * p.G + 2 * kTileRows - 1) / (2 * kTileRows);
+  if (n_ctas <= 0) return cudaSuccess;
+  if (D == 128) return launch_pair_t<128>(km, vm, p, n_ctas, s);
+  if (D == 64) return launch_pair_t<64>(km, vm, p, n_ctas, s);
   return cudaErrorInvalidValue;
 }
 

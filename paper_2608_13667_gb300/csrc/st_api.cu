@@ -10,6 +10,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -306,23 +307,38 @@ st_status flush_tables(st_pool* P, cudaStream_t s) {
 bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // Validates and performs an append (shared by st_append_kv and st_merge).
-st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const void* k, const void* v,
-                    cudaStream_t s) {
+// Appends counts[i] rows to slots[i], in order (the same page allocation as
+// appending to each sequence in turn); k, v: [L][sum of counts][Hkv][D].
+// All or nothing: capacity is checked before any table changes.
+st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, int n_br, const void* k,
+                         const void* v, cudaStream_t s) {
   BlockPool& bp = *P->pool;
-  int64_t need = 0;
+  int64_t need = 0, n_rows = 0;
+  bool uniform = true;
   for (int i = 0; i < n_br; ++i) {
-    if (!bp.fits(slots[i], n_tok))
+    if (!bp.fits(slots[i], counts[i]))
       return fail(P, ST_ERR_OOM, "sequence would exceed max_pages (%d)", bp.max_pages());
-    need += bp.pages_needed(slots[i], n_tok);
+    need += bp.pages_needed(slots[i], counts[i]);
+    n_rows += counts[i];
+    uniform = uniform && counts[i] == counts[0];
   }
   if (need > bp.free_count())
     return fail(P, ST_ERR_OOM, "pool has %lld free pages, call needs %lld",
                 (long long)bp.free_count(), (long long)need);
-  std::vector<int32_t> starts(n_br);
-  for (int i = 0; i < n_br; ++i) starts[i] = (int32_t)bp.slot(slots[i]).len;
+  if (n_rows > INT32_MAX) return fail(P, ST_ERR_INVALID, "too many rows in one call");
+  std::vector<AppendBranch> brs(n_br);
+  int32_t row0 = 0;
+  for (int i = 0; i < n_br; ++i) {
+    brs[i] = AppendBranch{slots[i], (int32_t)bp.slot(slots[i]).len, row0, counts[i]};
+    row0 += counts[i];
+  }
   std::vector<CowEvent> cows;
-  bp.append(slots, n_br, n_tok, &cows);
-  if (P->meta_only || n_tok == 0) return ST_OK;
+  if (uniform) {
+    bp.append(slots, n_br, n_br ? counts[0] : 0, &cows);
+  } else {
+    for (int i = 0; i < n_br; ++i) bp.append(&slots[i], 1, counts[i], &cows);
+  }
+  if (P->meta_only || n_rows == 0) return ST_OK;
 
   st_status st = flush_tables(P, s);
   if (st != ST_OK) return st;
@@ -334,7 +350,7 @@ st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const voi
   Plan plan;
   int ps = -1;
   if (inline_plan) {
-    for (int i = 0; i < n_br; ++i) inl.branches[i] = AppendBranch{slots[i], starts[i]};
+    for (int i = 0; i < n_br; ++i) inl.branches[i] = brs[i];
     for (size_t i = 0; i < cows.size(); ++i)
       inl.cows[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
   } else {
@@ -343,7 +359,7 @@ st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const voi
     AppendBranch* br = plan.alloc<AppendBranch>(n_br, &d_br);
     CowCopy* cw = plan.alloc<CowCopy>(std::max<size_t>(cows.size(), 1), &d_cow);
     if (!br || !cw) return fail(P, ST_ERR_INVALID, "append plan does not fit the staging slot");
-    for (int i = 0; i < n_br; ++i) br[i] = AppendBranch{slots[i], starts[i]};
+    for (int i = 0; i < n_br; ++i) br[i] = brs[i];
     for (size_t i = 0; i < cows.size(); ++i)
       cw[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
     st = submit_plan(P, plan, s);
@@ -362,18 +378,26 @@ st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const voi
   ap.n_blocks = c.n_blocks;
   ap.n_cow = (int32_t)cows.size();
   ap.n_br = n_br;
-  ap.n_tok = n_tok;
+  ap.n_tok = uniform && n_br ? counts[0] : 0;
   ap.L = c.n_layers;
   ap.Hkv = c.n_kv_heads;
   ap.max_pages = c.max_pages;
+  ap.n_rows = (int32_t)n_rows;
+  ap.ragged = uniform ? 0 : 1;
   const double row_bytes = (double)c.n_layers * c.n_kv_heads * c.head_dim * 2 * 2;
   double cow_rows = 0;
   for (auto& e : cows) cow_rows += e.rows;
-  const double bytes = row_bytes * ((double)n_br * n_tok * 2 + cow_rows * 2);
+  const double bytes = row_bytes * ((double)n_rows * 2 + cow_rows * 2);
   st = run_kernel(P, kKAppend, bytes, 0, s,
                   [&] { return launch_append(ap, inline_plan ? &inl : nullptr, c.head_dim, s); });
   if (st != ST_OK) return st;
   return inline_plan ? ST_OK : retire_plan(P, ps, s);
+}
+
+st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const void* k, const void* v,
+                    cudaStream_t s) {
+  std::vector<int32_t> counts(n_br, n_tok);
+  return do_append_rows(P, slots, counts.data(), n_br, k, v, s);
 }
 
 // Longest common prefix (in pages) of two block tables.
@@ -860,7 +884,92 @@ ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, con
   const double keys = (double)n_tok * L0 + (double)n_tok * (n_tok + 1) / 2;
   const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
   return run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
-                    [&] { return launch_merge_tc(P->kmap, P->vmap, ap, c.head_dim, s); });
+                    [&] { return launch_merge_tc(P->kmap, P->vmap, ap, 0, c.head_dim, s); });
+}
+
+ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, const int32_t* n_tok,
+                                  const void* q, const void* k, const void* v, float* o, float* lse,
+                                  void* stream) {
+  if (!P) return ST_ERR_INVALID;
+  if (n_seq < 0 || (n_seq > 0 && (!seqs || !n_tok))) return fail(P, ST_ERR_INVALID, "bad n_seq/seqs/n_tok");
+  std::vector<int> slots;
+  std::vector<int32_t> counts;
+  std::vector<int> all(n_seq);
+  int64_t R = 0;
+  for (int i = 0; i < n_seq; ++i) {
+    if (!decode_handle(P, seqs[i], &all[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+    for (int j = 0; j < i; ++j)
+      if (all[j] == all[i]) return fail(P, ST_ERR_INVALID, "sequence listed twice");
+    if (n_tok[i] < 0) return fail(P, ST_ERR_INVALID, "n_tok[%d] < 0", i);
+    if (n_tok[i] > 0) {
+      slots.push_back(all[i]);
+      counts.push_back(n_tok[i]);
+      R += n_tok[i];
+    }
+  }
+  if (R > INT32_MAX) return fail(P, ST_ERR_INVALID, "too many rows in one call");
+  if (P->meta_only) {
+    if (q || k || v || o || lse) return fail(P, ST_ERR_INVALID, "metadata-only pool takes no data");
+    return do_append_rows(P, slots.data(), counts.data(), (int)slots.size(), nullptr, nullptr, nullptr);
+  }
+  if (R == 0) return ST_OK;
+  if (!q || !k || !v || !o || !lse || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) ||
+      !aligned(o, 16) || !aligned(lse, 4))
+    return fail(P, ST_ERR_INVALID, "q/k/v/o/lse must be aligned device pointers");
+  const st_config& c = P->cfg;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  std::vector<int32_t> L0(slots.size());
+  for (size_t i = 0; i < slots.size(); ++i) L0[i] = (int32_t)P->pool->slot(slots[i]).len;
+  DeviceGuard guard(P->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  st_status st = do_append_rows(P, slots.data(), counts.data(), (int)slots.size(), k, v, s);
+  if (st != ST_OK) return st;
+
+  // work items: each sequence's stacked (row, head) rows in tiles of 256
+  std::vector<MergeItem> items;
+  double kv_bytes = 0, io_bytes = 0, keys = 0;
+  int32_t q_row0 = 0;
+  for (size_t i = 0; i < slots.size(); ++i) {
+    const int64_t rows = (int64_t)counts[i] * G;
+    for (int64_t rb = 0; rb < rows; rb += 256)
+      items.push_back(MergeItem{slots[i], L0[i], counts[i], q_row0, (int32_t)rb, {0, 0, 0}});
+    kv_bytes += (double)(L0[i] + counts[i]) * c.n_kv_heads * c.head_dim * 2 * 2 * c.n_layers;
+    keys += (double)counts[i] * L0[i] + (double)counts[i] * (counts[i] + 1) / 2;
+    q_row0 += counts[i];
+  }
+  io_bytes = (double)c.n_layers * R * c.n_q_heads * (c.head_dim * 2 + c.head_dim * 4 + 4);
+  const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
+  Plan plan;
+  int ps = -1;
+  st = acquire_plan(P, &plan, &ps);
+  if (st != ST_OK) return st;
+  const MergeItem* d_items = nullptr;
+  MergeItem* hi = plan.alloc<MergeItem>(items.size(), &d_items);
+  if (!hi) return fail(P, ST_ERR_INVALID, "prefill plan does not fit the staging slot");
+  std::memcpy(hi, items.data(), items.size() * sizeof(MergeItem));
+  st = submit_plan(P, plan, s);
+  if (st != ST_OK) return st;
+  AttnParams ap{};
+  ap.q = static_cast<const __nv_bfloat16*>(q);
+  ap.out_o = o;
+  ap.out_lse = lse;
+  ap.table = P->d_tables;
+  ap.status = P->d_status;
+  ap.n_blocks = c.n_blocks;
+  ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c.head_dim));
+  ap.n_rows_q = (int32_t)R;
+  ap.Hq = c.n_q_heads;
+  ap.Hkv = c.n_kv_heads;
+  ap.G = G;
+  ap.L = c.n_layers;
+  ap.max_pages = c.max_pages;
+  ap.max_splits = c.max_splits;
+  ap.mitems = d_items;
+  const int n_items = (int)items.size();
+  st = run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
+                  [&] { return launch_merge_tc(P->kmap, P->vmap, ap, n_items, c.head_dim, s); });
+  if (st != ST_OK) return st;
+  return retire_plan(P, ps, s);
 }
 
 ST_API st_status st_block_table(st_pool* P, st_seq seq, int32_t* out, int cap, int* n_pages,

@@ -95,6 +95,23 @@ class Run:
         self.hist[rid].append((tag, 0, T))
         return q, o, lse, L0
 
+    def prefill_batch(self, rids, counts, tag):
+        """Batched prefill: counts[i] rows onto rids[i], packed in that order."""
+        w = self.w
+        R = sum(counts)
+        k, v = kv_rows(w, tag, R, device=self.device)
+        q = queries(w, ("prefill_q",) + tuple(tag), R, device=self.device)
+        L0 = [self.ref.seqs[r].length for r in rids]
+        o, lse = self.pool.prefill_batch([self.handle[r] for r in rids], counts, q, k, v)
+        self.ref.prefill_batch(rids, counts)
+        self.sizes[tag] = R
+        off = 0
+        for r, n in zip(rids, counts):
+            if n:
+                self.hist[r].append((tag, off, n))
+            off += n
+        return q, o, lse, L0
+
     def release(self, rid):
         self.ref.release(rid)
         self.pool.release(self.handle[rid])

@@ -77,6 +77,21 @@ def test_random_traces_match_reference_bit_exactly(stlib, seed):
             else:
                 with pytest.raises(stlib.STError):
                     lp.merge(handles[m], T, None, None)
+        elif op < 0.82 and live:
+            # batched prefill: ragged counts (zeros included), sequences in order
+            ids = r.sample(live, r.randint(1, min(5, len(live))))
+            counts = [r.choice([0, 1, 5, 16, 17, 40]) for _ in ids]
+            try:
+                ref.prefill_batch(ids, counts)
+                ok = True
+            except R.OutOfBlocks:
+                ok = False
+            if ok:
+                lp.prefill_batch([handles[i] for i in ids], counts, None, None, None)
+            else:
+                with pytest.raises(stlib.STError) as e:
+                    lp.prefill_batch([handles[i] for i in ids], counts, None, None, None)
+                assert e.value.status == stlib.ST_ERR_OOM
         elif op < 0.9 and len(live) > 1:
             x = r.choice(live)
             ref.release(x)
