@@ -371,6 +371,67 @@ def _merge_case(n_merges=3):
             "merges": n_merges}
 
 
+def run_prefill_batch():
+    """Batched prefill on the batched-serving shape (1 layer, 32/8 heads, D 128):
+    16 agents with contexts of 4096-32768 tokens each receive an observation of
+    64-1024 rows (seeded).  One st_prefill_batch against one st_merge per agent
+    on a second, identical set of agents.  Prints CUDA-event timings."""
+    import numpy as np
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import get, kv_rows, queries
+    dev = torch.device("cuda", 0)
+    st.build()
+    w = get(3)
+    rng = np.random.default_rng(7)
+    obs = [int(x) for x in rng.integers(64, 1024, size=w.n_tasks, endpoint=True)]
+    pages = 2 * sum((p + n + 15) // 16 + 1 for p, n in zip(w.prefix, obs))
+    pool = st.Pool(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads, head_dim=w.head_dim,
+                   n_blocks=pages + 64, seed=w.seed, device=dev, max_seqs=2 * w.n_tasks + 3,
+                   max_pages=max(w.prefix) // 16 + 80, max_decode_branches=8, max_splits=8)
+    sets = []
+    for rep in range(2):
+        seqs = []
+        for t_, p in enumerate(w.prefix):
+            m = pool.seq_create()
+            k, v = kv_rows(w, ("prefix", t_), p, device=dev)
+            pool.append_kv([m], k.view(w.n_layers, 1, p, w.n_kv_heads, w.head_dim),
+                           v.view(w.n_layers, 1, p, w.n_kv_heads, w.head_dim))
+            seqs.append(m)
+        sets.append(seqs)
+    R = sum(obs)
+    k, v = kv_rows(w, ("obs",), R, device=dev)
+    q = queries(w, ("obs_q",), R, device=dev)
+    # warm-up on a small extra sequence (first-launch setup stays out of the timings)
+    x = pool.seq_create()
+    pool.append_kv([x], k[:, :64].contiguous().view(w.n_layers, 1, 64, w.n_kv_heads, w.head_dim),
+                   v[:, :64].contiguous().view(w.n_layers, 1, 64, w.n_kv_heads, w.head_dim))
+    pool.merge(x, q[:, :16].contiguous(), k[:, :16].contiguous(), v[:, :16].contiguous())
+    pool.prefill_batch([x], [16], q[:, :16].contiguous(), k[:, :16].contiguous(), v[:, :16].contiguous())
+    keys = sum(n * p + n * (n + 1) / 2 for p, n in zip(w.prefix, obs))
+    flops = 4.0 * w.head_dim * keys * w.n_q_heads * w.n_layers
+    pool.sync()
+    pool.profile_read()
+    pool.profile_enable(True)
+    pool.prefill_batch(sets[0], obs, q, k, v)
+    pool.sync()
+    b = pool.profile_read()
+    off = 0
+    for m, n in zip(sets[1], obs):
+        pool.merge(m, q[:, off:off + n].contiguous(), k[:, off:off + n].contiguous(), v[:, off:off + n].contiguous())
+        off += n
+    pool.sync()
+    s_ = pool.profile_read()
+    pool.close()
+    bm, sm_ = b["merge_prefill"], s_["merge_prefill"]
+    ba, sa = b["append_kv"], s_["append_kv"]
+    print(json.dumps({"agents": w.n_tasks, "rows": R, "tflop": flops / 1e12,
+                      "batched": {"launches": bm["launches"], "prefill_ms": bm["total_ms"],
+                                  "append_ms": ba["total_ms"], "tflops": flops / bm["total_ms"] / 1e9},
+                      "per_agent": {"launches": sm_["launches"], "prefill_ms": sm_["total_ms"],
+                                    "append_ms": sa["total_ms"], "tflops": flops / sm_["total_ms"] / 1e9}}))
+
+
 def run_profile_merge():
     """Only the merge case of run_profile_small (about 1 GB on the device):
     three identical merge launches, for ncu captures of the merge kernel."""
@@ -522,6 +583,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-small", action="store_true",
                     help="run the small decode + merge case used for ncu captures and exit")
+    ap.add_argument("--prefill-batch", action="store_true",
+                    help="time one batched prefill of 16 agents against one merge per agent and exit")
     ap.add_argument("--profile-merge", action="store_true",
                     help="run only the merge case of --profile-small (three identical launches) and exit")
     ap.add_argument("--cycle", action="store_true",
@@ -532,6 +595,9 @@ def main():
         return
     if args.profile_merge:
         run_profile_merge()
+        return
+    if args.prefill_batch:
+        run_prefill_batch()
         return
     if args.cycle:
         run_cycle()
