@@ -371,6 +371,38 @@ def _merge_case(n_merges=3):
             "merges": n_merges}
 
 
+def run_profile_wide():
+    """The wide decode tile on a small case for ncu captures: the long-trajectory
+    decode with 9 branches per group (72 stacked rows) and 4 layers instead of 32,
+    three decode steps.  Prints the CUDA-event timing of the last one."""
+    import dataclasses
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import kv_rows, queries
+    from workloads.configs import long_with_branches
+    dev = torch.device("cuda", 0)
+    st.build()
+    w = dataclasses.replace(long_with_branches(8), n_layers=4)
+    pool, br = build_long_workload(w, dev)
+    n = len(br)
+    o = torch.empty((w.n_layers, n, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+    lse = torch.empty((w.n_layers, n, w.n_q_heads), dtype=torch.float32, device=dev)
+    for s in range(3):
+        k, v = kv_rows(w, ("step", s), n, device=dev)
+        shape = (w.n_layers, n, 1, w.n_kv_heads, w.head_dim)
+        pool.append_kv(br, k.view(shape), v.view(shape))
+        if s == 2:  # time the last step alone
+            pool.sync()
+            pool.profile_read()
+            pool.profile_enable(True)
+        pool.decode_attn(br, queries(w, ("q", s), n, device=dev), o, lse)
+    pool.sync()
+    d = pool.profile_read()["decode_partial"]
+    pool.close()
+    print(json.dumps({"workload": w.name, "layers": w.n_layers, "decode_ms": d["total_ms"] / d["launches"],
+                      "decode_gbs": d["bytes"] / d["total_ms"] / 1e6}))
+
+
 def run_prefill_batch():
     """Batched prefill on the batched-serving shape (1 layer, 32/8 heads, D 128):
     16 agents with contexts of 4096-32768 tokens each receive an observation of
@@ -583,6 +615,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-small", action="store_true",
                     help="run the small decode + merge case used for ncu captures and exit")
+    ap.add_argument("--profile-wide", action="store_true",
+                    help="run the small 9-branch decode case (wide tile) used for ncu captures and exit")
     ap.add_argument("--prefill-batch", action="store_true",
                     help="time one batched prefill of 16 agents against one merge per agent and exit")
     ap.add_argument("--profile-merge", action="store_true",
@@ -598,6 +632,9 @@ def main():
         return
     if args.prefill_batch:
         run_prefill_batch()
+        return
+    if args.profile_wide:
+        run_profile_wide()
         return
     if args.cycle:
         run_cycle()
