@@ -19,6 +19,8 @@
 #include <tuple>
 #include <new>
 #include <string>
+
+#include <nvtx3/nvToolsExt.h>
 #include <vector>
 
 #include "../../include/st.h"
@@ -553,7 +555,17 @@ ST_API st_status st_seq_create(st_pool* P, st_seq* out) {
   return ST_OK;
 }
 
+// NVTX range around each public call that issues work (no cost unless a
+// profiler is attached), so that ncu / nsys can filter by call.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 ST_API st_status st_fork(st_pool* P, st_seq seq, int n_aux, st_seq* out_aux) {
+  NvtxRange range_("st_fork");
   if (!P) return ST_ERR_INVALID;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
@@ -561,6 +573,7 @@ ST_API st_status st_fork(st_pool* P, st_seq seq, int n_aux, st_seq* out_aux) {
 }
 
 ST_API st_status st_fork_at(st_pool* P, st_seq seq, int64_t length, int n_aux, st_seq* out_aux) {
+  NvtxRange range_("st_fork_at");
   if (!P) return ST_ERR_INVALID;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
@@ -577,6 +590,7 @@ ST_API st_status st_fork_at(st_pool* P, st_seq seq, int64_t length, int n_aux, s
 }
 
 ST_API st_status st_release(st_pool* P, st_seq seq) {
+  NvtxRange range_("st_release");
   if (!P) return ST_ERR_INVALID;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
@@ -586,6 +600,7 @@ ST_API st_status st_release(st_pool* P, st_seq seq) {
 
 ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok, const void* k,
                               const void* v, void* stream) {
+  NvtxRange range_("st_append_kv");
   if (!P) return ST_ERR_INVALID;
   if (n_br < 0 || n_tok < 0 || (n_br > 0 && !br)) return fail(P, ST_ERR_INVALID, "bad n_br/n_tok");
   std::vector<int> slots(n_br);
@@ -606,6 +621,7 @@ ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok,
 
 ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const void* q, float* o,
                                 float* lse, void* stream) {
+  NvtxRange range_("st_decode_attn");
   if (!P) return ST_ERR_INVALID;
   if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
   if (n_br < 1 || !br) return fail(P, ST_ERR_INVALID, "need at least one branch");
@@ -841,6 +857,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
 
 ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, const void* k,
                           const void* v, float* o, float* lse, void* stream) {
+  NvtxRange range_("st_merge");
   if (!P) return ST_ERR_INVALID;
   int slot;
   if (!decode_handle(P, main, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
@@ -890,6 +907,7 @@ ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, con
 ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, const int32_t* n_tok,
                                   const void* q, const void* k, const void* v, float* o, float* lse,
                                   void* stream) {
+  NvtxRange range_("st_prefill_batch");
   if (!P) return ST_ERR_INVALID;
   if (n_seq < 0 || (n_seq > 0 && (!seqs || !n_tok))) return fail(P, ST_ERR_INVALID, "bad n_seq/seqs/n_tok");
   std::vector<int> slots;
@@ -1005,6 +1023,7 @@ ST_API st_status st_free_list(st_pool* P, int32_t* out, int64_t cap, int64_t* n)
 }
 
 ST_API st_status st_sync(st_pool* P, void* stream) {
+  NvtxRange range_("st_sync");
   if (!P) return ST_ERR_INVALID;
   if (P->meta_only) return ST_OK;
   DeviceGuard guard(P->device);
