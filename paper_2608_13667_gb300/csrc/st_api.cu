@@ -706,11 +706,39 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     total_pages += own_pages[i];
   }
   const int64_t units = total_pages * c.n_kv_heads * c.n_layers;
-  const int64_t target_ctas = (int64_t)32 * P->sms * P->decode_ctas_per_sm;
+  const int64_t slots_per_wave = (int64_t)P->sms * P->decode_ctas_per_sm;
+  const int64_t target_ctas = 32 * slots_per_wave;
   int64_t chunk = (units + target_ctas - 1) / target_ctas;
   chunk = std::max<int64_t>(16, (chunk + 3) / 4 * 4);
   // leave room for a branch's own runs, but never fewer than one run for the prefix
   const int max_prefix_chunks = std::max(1, c.max_splits - 2);
+  // CTAs the runs of a given length make (the items below, times heads and layers)
+  auto ctas_for = [&](int64_t ch) {
+    int64_t n = 0;
+    std::vector<int32_t> ns(n_br, 0);
+    for (auto& g : groups) {
+      const int64_t k = std::min<int64_t>(max_prefix_chunks, (g.pages + ch - 1) / ch);
+      n += k;
+      for (int i : g.members) ns[i] = (int32_t)k;
+    }
+    for (int i = 0; i < n_br; ++i)
+      if (own_pages[i] > 0) n += std::min<int64_t>(c.max_splits - ns[i], (own_pages[i] + ch - 1) / ch);
+    return n * c.n_kv_heads * c.n_layers;
+  };
+  // A small launch (a few waves) whose last wave is less than half full: longer
+  // runs (whole 4-page stages at a time) until a wave disappears, since a wave
+  // costs a CTA's whole latency however few CTAs are in it.
+  {
+    const int64_t n0 = ctas_for(chunk), waves = (n0 + slots_per_wave - 1) / slots_per_wave;
+    if (waves <= 4 && n0 % slots_per_wave != 0 && n0 % slots_per_wave < slots_per_wave / 2) {
+      for (int64_t ch = chunk + 4; ch <= chunk + 64; ch += 4) {
+        if ((ctas_for(ch) + slots_per_wave - 1) / slots_per_wave < waves) {
+          chunk = ch;
+          break;
+        }
+      }
+    }
+  }
 
   st_status st = flush_tables(P, s);
   if (st != ST_OK) return st;
