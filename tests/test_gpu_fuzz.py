@@ -1,6 +1,6 @@
 """Randomised parity sweep: random geometries, split budgets, fork points,
-group mixes and step counts, every decode and merge checked against the
-float64 oracle, tables and refcounts checked bit-exactly."""
+group mixes and step counts, every decode, merge and batched prefill checked
+against the float64 oracle, tables and refcounts checked bit-exactly."""
 import numpy as np
 import pytest
 
@@ -56,5 +56,18 @@ def test_random_fork_groups(stlib, seed):
     k, v = run.context(m, layer)
     o_ref, l_ref = A.merge_prefill(qm[layer].cpu(), k, v, L0)
     compare(om[layer], lm[layer], o_ref, l_ref, f"seed {seed} merge")
+    # a batched prefill over a random subset (ragged counts, zeros included)
+    sub = [rids[i] for i in sorted(rng.choice(len(rids), size=int(rng.integers(1, len(rids) + 1)),
+                                              replace=False))]
+    counts = [int(rng.choice([0, 1, 9, 16, 17, 40, 77])) for _ in sub]
+    qp, op, lp, L0s = run.prefill_batch(sub, counts, ("batch",))
+    layer = int(rng.integers(0, L))
+    off = 0
+    for r, n, l0 in zip(sub, counts, L0s):
+        if n:
+            k, v = run.context(r, layer)
+            o_ref, l_ref = A.merge_prefill(qp[layer, off:off + n].cpu(), k, v, l0)
+            compare(op[layer, off:off + n], lp[layer, off:off + n], o_ref, l_ref, f"seed {seed} batch seq {r}")
+        off += n
     run.pool.sync()
     run.check_tables()
