@@ -7,7 +7,9 @@
 // head are stacked G per token; a CTA takes 256 consecutive stacked rows as
 // tile A (the first 128) and tile B (the next 128) and walks main's pages up
 // to the causal limit of its last row, 128 keys per stage.  Both tiles read
-// each K/V stage from shared memory.
+// each K/V stage from shared memory.  A batched prefill (several sequences'
+// new rows in one launch) gives each CTA its own (sequence, L0, T, row tile)
+// through a work list.
 //
 // CTA layout (352 threads, one CTA per SM, all 512 TMEM columns):
 //   warps 0..3  softmax of tile A, warps 4..7 softmax of tile B: thread r of
@@ -22,7 +24,9 @@
 //   warp 8      K loader, warp 9 V loader: page ids from the block table (32
 //               per read, one batch ahead), one 2 KiB TMA copy per (page,
 //               64-wide half of D) into separate K and V rings.
-//   warp 10     TMEM owner; lane 0 issues, per stage j and tile t = A, B,
+//   warp 10     TMEM owner and MMA issuer (the whole warp runs the loop with
+//               warp-uniform operands, an elected lane issues), per stage j
+//               and tile t = A, B,
 //                 O_t += P_t(j-1) V_{j-1}   (A = P_hi, P_lo from TMEM, M 128, N D)
 //                 S_t(j) = Q_t K_j^T        (M 128, N 128)
 //               so that the softmax of one tile overlaps the MMAs of the
