@@ -927,6 +927,7 @@ ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, con
   ap.slot = slot;
   ap.L0 = (int32_t)L0;
   ap.T = n_tok;
+  ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
   // algorithmic: main's KV once per (layer, head) + Q + O/LSE; flops: causal
   const double kv_bytes = (double)(L0 + n_tok) * c.n_kv_heads * c.head_dim * 2 * 2 * c.n_layers;
   const double io_bytes = (double)c.n_layers * n_tok * c.n_q_heads * (c.head_dim * 2 + c.head_dim * 4 + 4);
@@ -1015,6 +1016,7 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
   ap.max_pages = c.max_pages;
   ap.max_splits = c.max_splits;
   ap.mitems = d_items;
+  ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
   const int n_items = (int)items.size();
   st = run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
                   [&] { return launch_merge_tc(P->kmap, P->vmap, ap, n_items, c.head_dim, s); });

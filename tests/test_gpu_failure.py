@@ -1,8 +1,8 @@
-"""The device-timeout path: every wait in the attention kernel is bounded.
+"""The device-timeout path: every wait in the attention kernels is bounded.
 With the ST_FLAG_HOLD_LOADS test hook nothing ever arrives on the decode's
-stage barriers; the waits run out (2 s), the kernel records ST_ERR_TIMEOUT
-and returns without faulting, st_sync reports it, and the context stays
-usable for a normal pool afterwards."""
+or the merge's stage barriers; the waits run out (2 s), the kernel records
+ST_ERR_TIMEOUT and returns without faulting, st_sync reports it, and the
+context stays usable for a normal pool afterwards."""
 import time
 
 import pytest
@@ -39,3 +39,35 @@ def test_decode_wait_runs_out_and_is_reported(stlib):
     run.pool.sync()
     o_ref, l_ref = run.oracle_decode([b], q2, 0)
     compare(o[0], lse[0], o_ref, l_ref, "after timeout")
+
+
+@pytest.mark.parametrize("batched", [False, True])
+def test_merge_wait_runs_out_and_is_reported(stlib, batched):
+    w = Workload(name="holdm", n_layers=1, n_q_heads=8, n_kv_heads=2, head_dim=64, n_blocks=64, seed=43)
+    pool = stpkg.Pool(n_layers=1, n_q_heads=8, n_kv_heads=2, head_dim=64, n_blocks=64, seed=43,
+                      max_seqs=2, max_decode_branches=1, max_splits=2, flags=stpkg.ST_FLAG_HOLD_LOADS)
+    a = pool.seq_create()
+    k, v = kv_rows(w, ("ctx",), 40, device="cuda")
+    pool.append_kv([a], k.view(1, 1, 40, 2, 64), v.view(1, 1, 40, 2, 64))
+    km, vm = kv_rows(w, ("m",), 10, device="cuda")
+    qm = queries(w, ("mq",), 10, device="cuda")
+    t0 = time.time()
+    if batched:
+        pool.prefill_batch([a], [10], qm, km, vm)
+    else:
+        pool.merge(a, qm, km, vm)            # two CTAs (one per KV head): their waits run out
+    with pytest.raises(stpkg.STError) as e:
+        pool.sync()
+    assert e.value.status == stpkg.ST_ERR_TIMEOUT
+    assert time.time() - t0 < 60
+    pool.sync()
+    pool.close()
+    run = Run(w, max_seqs=2, max_decode_branches=1, max_splits=2)
+    b = run.create()
+    run.append([b], 40, ("ctx2",))
+    qm2, om, lm, L0 = run.merge(b, 10, ("m2",))
+    run.pool.sync()
+    from oracle import attention as A
+    kk, vv = run.context(b, 0)
+    o_ref, l_ref = A.merge_prefill(qm2[0].cpu(), kk, vv, L0)
+    compare(om[0], lm[0], o_ref, l_ref, "merge after timeout")
