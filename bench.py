@@ -241,24 +241,32 @@ def run_ours(args, rank, ws, local):
 
     # end-to-end through the public API with host buffers: H2D of the step's
     # q and new K/V rows from pinned memory, D2H of O and LSE, every step
-    e2e_steps = max(2, min(args.steps, 5))
-    hq = [step_q[s % n_steps].cpu().pin_memory() for s in range(e2e_steps)]
-    hk = [step_k[s % n_steps].cpu().pin_memory() for s in range(e2e_steps)]
-    hv = [step_v[s % n_steps].cpu().pin_memory() for s in range(e2e_steps)]
+    e2e_steps = max(2, min(args.steps, 10))
+    e2e_warm = 2  # first use of the pinned buffers stays out of the timing
+    n_host = min(e2e_steps, 4)  # distinct host input sets, used in turn
+    hq = [step_q[s % n_steps].cpu().pin_memory() for s in range(n_host)]
+    hk = [step_k[s % n_steps].cpu().pin_memory() for s in range(n_host)]
+    hv = [step_v[s % n_steps].cpu().pin_memory() for s in range(n_host)]
     ho = torch.empty(o.shape, dtype=o.dtype).pin_memory()
     hl = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
     dq, dk, dv = torch.empty_like(step_q[0]), torch.empty_like(step_k[0]), torch.empty_like(step_v[0])
-    _barrier(ws)
-    torch.cuda.synchronize(dev)
-    t0 = time.perf_counter()
-    for s in range(e2e_steps):
-        dq.copy_(hq[s], non_blocking=True)
-        dk.copy_(hk[s], non_blocking=True)
-        dv.copy_(hv[s], non_blocking=True)
+
+    def e2e_step(s):
+        dq.copy_(hq[s % n_host], non_blocking=True)
+        dk.copy_(hk[s % n_host], non_blocking=True)
+        dv.copy_(hv[s % n_host], non_blocking=True)
         pool.append_kv(br, dk, dv)
         pool.decode_attn(br, dq, o, lse)
         ho.copy_(o, non_blocking=True)
         hl.copy_(lse, non_blocking=True)
+
+    for s in range(e2e_warm):
+        e2e_step(s)
+    _barrier(ws)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for s in range(e2e_steps):
+        e2e_step(s)
     torch.cuda.synchronize(dev)
     e2e_s = _allreduce_max(time.perf_counter() - t0, ws)
     h2d = hq[0].numel() * 2 + hk[0].numel() * 2 * 2

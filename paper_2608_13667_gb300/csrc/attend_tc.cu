@@ -81,6 +81,10 @@ struct TcCfg {
   static constexpr int kKeys = 64;                     // keys per stage
   static constexpr int kPagesPerStage = kKeys / kPageTokens;
   static constexpr int kStages = kWide ? 2 : 3;
+  // Wide: P lives in TMEM, so a K slot is free once S_j has been computed and
+  // K and V slots recycle separately (K and V barrier rings); narrow: P goes
+  // over K_j, the two are released together after P_j V_j
+  static constexpr bool kSplitKV = kWide;
   // MMA M = 64 for <= 48 stacked rows: accumulator rows sit in TMEM lanes
   // 0..15 of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
   // M = 128 for up to 128 rows (row r at lane r)
@@ -117,14 +121,16 @@ __global__ void __launch_bounds__(kThreads, 2)
   uint8_t* q_s = base;
   uint8_t* ring = base + C::kQBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::kBarOffset);
-  uint64_t* full = bars;                 // [kStages]
-  uint64_t* empty = bars + C::kStages;   // [kStages]
+  uint64_t* full = bars;                 // [kStages] K (and, narrow, V) landed
+  uint64_t* empty = bars + C::kStages;   // [kStages] K (and, narrow, V) slot free
   uint64_t* s_full = bars + 2 * C::kStages;   // [2] per S buffer
   uint64_t* p_full = s_full + 2;              // [2] per S buffer
   uint64_t* o_ready = s_full + 4;             // one phase per P V
   uint64_t* o_final = s_full + 5;
   uint64_t* q_ready = s_full + 6;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 7);
+  uint64_t* v_full = s_full + 8;               // [kStages] wide: V landed
+  uint64_t* v_empty = v_full + C::kStages;     // [kStages] wide: V slot free
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -149,6 +155,10 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
+      if (C::kSplitKV) {
+        mbar_init(&v_full[s], 1);
+        mbar_init(&v_empty[s], 1);
+      }
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&s_full[b], 1);
@@ -179,19 +189,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
     int nxt = 32 + lane < n_pages ? ids[32 + lane] : 0;
-    int j = 0;
-    bool ok = true;
-    for (; j < n_tiles; ++j) {
-      const int s = j % C::kStages;
-      if (j >= C::kStages) {
-        int w = 1;
-        if (lane == 0) w = mbar_wait(&empty[s], ((j / C::kStages) - 1) & 1) ? 1 : 0;
-        w = __shfl_sync(0xffffffffu, w, 0);
-        if (!w) {
-          ok = false;
-          break;
-        }
-      }
+    // waits for slot s of a ring to be released for stage j (lane 0 waits)
+    auto slot_free = [&](uint64_t* ring_empty, int s, int j) -> bool {
+      int w = 1;
+      if (j >= C::kStages && lane == 0) w = mbar_wait(&ring_empty[s], ((j / C::kStages) - 1) & 1) ? 1 : 0;
+      return __shfl_sync(0xffffffffu, w, 0) != 0;
+    };
+    // pages of stage j (j increasing): the count and the TMA page coordinates
+    auto stage_pages = [&](int j, int* c3) -> int {
       const int page0 = j * C::kPagesPerStage;
       if (page0 >= base_id + 32) {
         base_id += 32;
@@ -199,34 +204,91 @@ __global__ void __launch_bounds__(kThreads, 2)
         nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
       }
       const int np = min(C::kPagesPerStage, n_pages - page0);
-      int blk[C::kPagesPerStage];
+#pragma unroll
+      for (int q = 0; q < C::kPagesPerStage; ++q) {
+        int b = __shfl_sync(0xffffffffu, cur, (page0 - base_id + q) & 31);
+        if (q < np && (uint64_t)b >= (uint64_t)p.n_blocks) {
+          if (lane == 0) atomicCAS(p.status, 0, kDevBadIndex);
+          b = 0;
+        }
+        c3[q] = layer * (int)p.n_blocks + b;
+      }
+      return np;
+    };
+    // wide: np pages of one operand into a slot, completing on bar (lane 0 issues)
+    const uint32_t page_bytes = (uint32_t)(C::kHalves * kPageTokens * 128);
+    auto issue = [&](const CUtensorMap* map, uint8_t* dst, uint64_t* bar, const int* c3, int np) {
+      if (lane != 0) return;
 #pragma unroll
       for (int q = 0; q < C::kPagesPerStage; ++q)
-        blk[q] = __shfl_sync(0xffffffffu, cur, (page0 - base_id + q) & 31);
-      if (lane == 0) {
-        uint8_t* kst = ring + s * C::kStageBytes;
-        uint8_t* vst = kst + C::kKSlotBytes;
-        mbar_arrive_expect_tx(&full[s], (uint32_t)(np * 2 * C::kHalves * kPageTokens * 128));
-        for (int q = 0; q < np; ++q) {
-          int b = blk[q];
-          if ((uint64_t)b >= (uint64_t)p.n_blocks) {
-            atomicCAS(p.status, 0, kDevBadIndex);
-            b = 0;
-          }
-          const int c3 = layer * (int)p.n_blocks + b;
 #pragma unroll
-          for (int h = 0; h < C::kHalves; ++h) {
-            tma_load_4d(kst + h * C::kKVHalfBytes + q * kPageTokens * 128, &kmap, &full[s], 0, h,
-                        kvh * kPageTokens, c3, policy);
-            tma_load_4d(vst + h * C::kKVHalfBytes + q * kPageTokens * 128, &vmap, &full[s], 0, h,
-                        kvh * kPageTokens, c3, policy);
+        for (int h = 0; h < C::kHalves; ++h)
+          if (q < np)
+            tma_load_4d(dst + h * C::kKVHalfBytes + q * kPageTokens * 128, map, bar, 0, h, kvh * kPageTokens,
+                        c3[q], policy);
+    };
+    int jk = 0, jv = 0;  // stages whose K and V copies have been issued
+    bool ok = true;
+    for (; jk < n_tiles; ++jk) {
+      const int s = jk % C::kStages;
+      if (!slot_free(empty, s, jk)) {
+        ok = false;
+        break;
+      }
+      uint8_t* kst = ring + s * C::kStageBytes;
+      uint8_t* vst = kst + C::kKSlotBytes;
+      if constexpr (C::kSplitKV) {
+        int c3[C::kPagesPerStage];
+        const int np = stage_pages(jk, c3);
+        if (lane == 0) mbar_arrive_expect_tx(&full[s], np * page_bytes);
+        issue(&kmap, kst, &full[s], c3, np);
+        // the K slot was released by S_j-kStages, the V slot waits for P_j-kStages V_j-kStages
+        if (!slot_free(v_empty, s, jk)) {
+          ok = false;
+          ++jk;  // K_j is in flight
+          break;
+        }
+        if (lane == 0) mbar_arrive_expect_tx(&v_full[s], np * page_bytes);
+        issue(&vmap, vst, &v_full[s], c3, np);
+        jv = jk + 1;
+      } else {
+        const int page0 = jk * C::kPagesPerStage;
+        if (page0 >= base_id + 32) {
+          base_id += 32;
+          cur = nxt;
+          nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
+        }
+        const int np = min(C::kPagesPerStage, n_pages - page0);
+        int blk[C::kPagesPerStage];
+#pragma unroll
+        for (int q = 0; q < C::kPagesPerStage; ++q)
+          blk[q] = __shfl_sync(0xffffffffu, cur, (page0 - base_id + q) & 31);
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&full[s], 2 * np * page_bytes);
+          for (int q = 0; q < np; ++q) {
+            int b = blk[q];
+            if ((uint64_t)b >= (uint64_t)p.n_blocks) {
+              atomicCAS(p.status, 0, kDevBadIndex);
+              b = 0;
+            }
+            const int c3 = layer * (int)p.n_blocks + b;
+#pragma unroll
+            for (int h = 0; h < C::kHalves; ++h) {
+              tma_load_4d(kst + h * C::kKVHalfBytes + q * kPageTokens * 128, &kmap, &full[s], 0, h,
+                          kvh * kPageTokens, c3, policy);
+              tma_load_4d(vst + h * C::kKVHalfBytes + q * kPageTokens * 128, &vmap, &full[s], 0, h,
+                          kvh * kPageTokens, c3, policy);
+            }
           }
         }
       }
     }
     if (!ok && lane == 0) {
       atomicCAS(p.status, 0, kDevTimeout);
-      for (int t = max(0, j - C::kStages); t < j; ++t) mbar_wait(&full[t % C::kStages], (t / C::kStages) & 1);
+      // wait (bounded) for this CTA's copies still in flight before it exits
+      for (int t = max(0, jk - C::kStages); t < jk; ++t) mbar_wait(&full[t % C::kStages], (t / C::kStages) & 1);
+      if constexpr (C::kSplitKV)
+        for (int t = max(0, jv - C::kStages); t < jv; ++t) mbar_wait(&v_full[t % C::kStages], (t / C::kStages) & 1);
     }
     return;
   }
@@ -254,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                         tc_desc_sw128(k_addr + h * C::kKVHalfBytes + kk * 32, 16, 1024), idesc_s,
                         (h | kk) != 0);
         tc_commit(&s_full[j & 1]);
+        if constexpr (C::kSplitKV) tc_commit(&empty[s]);  // K_j has been read
         return true;
       };
       if (ok) ok = issue_s(0);
@@ -280,6 +343,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint32_t k_addr = smem_addr(ring + s * C::kStageBytes);
         const uint32_t v_addr = k_addr + C::kKSlotBytes;
         if constexpr (kWide) {
+          if (!mbar_wait(&v_full[s], (j / C::kStages) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
           // P_hi, P_lo of keys [16 ks, 16 ks + 16) in the 16 TMEM columns of their scores
           const uint32_t p_tm = tmem + kTmemS + (j & 1) * C::kKeys;
 #pragma unroll
@@ -299,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
                         tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
         }
-        tc_commit(&empty[s]);
+        tc_commit(C::kSplitKV ? &v_empty[s] : &empty[s]);
         tc_commit(o_ready);
         if (jn < n_tiles && !early && !issue_s(jn)) {
           ok = false;
@@ -463,9 +531,12 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
     }
     if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
-      // this stage's copies have landed (S_j was computed from them): zero
-      // the V rows of keys that are not valid
-      mbar_wait(&full[s], (j / C::kStages) & 1);
+      // zero the V rows of keys that are not valid, once V_j has landed
+      // (narrow: with K_j, from which S_j was computed)
+      if (!__all_sync(0xffffffffu, mbar_wait(C::kSplitKV ? &v_full[s] : &full[s], (j / C::kStages) & 1))) {
+        ok = false;
+        break;
+      }
       uint8_t* vslot = kslot + C::kKSlotBytes;
       for (int t = tid; t < C::kKeys * C::kHalves; t += n_swt) {
         const int c = t % C::kKeys, h = t / C::kKeys;
