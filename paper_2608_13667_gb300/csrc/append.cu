@@ -14,6 +14,8 @@ namespace {
 
 __global__ void table_update_kernel(int32_t* __restrict__ table, const TableRun* __restrict__ runs,
                                     const int32_t* __restrict__ values, int n_runs) {
+  griddep_wait();
+  griddep_launch_dependents();
   for (int r = blockIdx.x; r < n_runs; r += gridDim.x) {
     const TableRun run = runs[r];
     for (int i = threadIdx.x; i < run.count; i += blockDim.x) table[run.dst + i] = values[run.src + i];
@@ -27,6 +29,8 @@ __global__ void table_update_kernel(int32_t* __restrict__ table, const TableRun*
 template <int D>
 __global__ void __launch_bounds__(256) append_kernel(const AppendParams p,
                                                      const __grid_constant__ InlineAppendPlan inl) {
+  griddep_wait();
+  griddep_launch_dependents();
   const AppendBranch* branches = p.branches ? p.branches : inl.branches;
   const CowCopy* cows = p.cows ? p.cows : inl.cows;
   constexpr int kChunks = D / 8;
@@ -104,8 +108,7 @@ cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int3
                                 int n_runs, cudaStream_t s) {
   if (n_runs <= 0) return cudaSuccess;
   const int grid = n_runs < 1024 ? n_runs : 1024;
-  table_update_kernel<<<grid, 256, 0, s>>>(table, runs, values, n_runs);
-  return cudaGetLastError();
+  return launch_chained(table_update_kernel, dim3(grid), dim3(256), 0, s, table, runs, values, n_runs);
 }
 
 cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, int D, cudaStream_t s) {
@@ -115,13 +118,9 @@ cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, in
                         (int64_t)p.L * p.n_rows * p.Hkv * (D / 8);
   if (total == 0) return cudaSuccess;
   const int grid = grid_for(total, 256);
-  if (D == 128)
-    append_kernel<128><<<grid, 256, 0, s>>>(p, ip);
-  else if (D == 64)
-    append_kernel<64><<<grid, 256, 0, s>>>(p, ip);
-  else
-    return cudaErrorInvalidValue;
-  return cudaGetLastError();
+  if (D == 128) return launch_chained(append_kernel<128>, dim3(grid), dim3(256), 0, s, p, ip);
+  if (D == 64) return launch_chained(append_kernel<64>, dim3(grid), dim3(256), 0, s, p, ip);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace st

@@ -137,6 +137,11 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int kvh = blockIdx.y;
   const int layer = blockIdx.z;
   const int G = p.G;
+  // the tensor-memory allocation touches no global memory: ahead of the wait
+  // for the previous kernel in the stream (the append that wrote the pages)
+  if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
+  griddep_wait();
+  griddep_launch_dependents();
 
   // ---- what this CTA reads and for whom ------------------------------------------
   const int32_t* members = p.members ? p.members : inl.members;
@@ -169,7 +174,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     mbar_init(q_ready, n_swt);
     fence_mbar_init();
   }
-  if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
@@ -599,8 +603,7 @@ cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const Attn
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  attend_tc_kernel<D, kWide><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
-  return cudaGetLastError();
+  return launch_chained(attend_tc_kernel<D, kWide>, grid, dim3(kThreads), C::kSmemBytes, s, km, vm, p, inl);
 }
 
 template <int D>

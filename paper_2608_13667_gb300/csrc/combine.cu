@@ -18,6 +18,8 @@ namespace {
 template <int D>
 __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
                                                       const __grid_constant__ InlineDecodePlan inl) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int32_t* n_splits = p.n_splits ? p.n_splits : inl.n_splits;
   const int lane = threadIdx.x & 31;
   const int64_t idx = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
@@ -88,13 +90,9 @@ cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, 
   const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
   if (total == 0) return cudaSuccess;
   const int grid = (int)((total + 3) / 4);
-  if (D == 128)
-    combine_kernel<128><<<grid, 128, 0, s>>>(p, ip);
-  else if (D == 64)
-    combine_kernel<64><<<grid, 128, 0, s>>>(p, ip);
-  else
-    return cudaErrorInvalidValue;
-  return cudaGetLastError();
+  if (D == 128) return launch_chained(combine_kernel<128>, dim3(grid), dim3(128), 0, s, p, ip);
+  if (D == 64) return launch_chained(combine_kernel<64>, dim3(grid), dim3(128), 0, s, p, ip);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace st

@@ -128,6 +128,38 @@ struct InlineAppendPlan {
   CowCopy cows[kInlineCows];
 };
 
+// Programmatic dependent launch.  The small kernels of a decode step (table
+// update, append, decode partials, combine) are launched so that each may be
+// scheduled while its predecessor in the stream is still running: it does
+// its setup that touches no global memory (barrier init, tensor-memory
+// allocation), then griddep_wait() blocks until the predecessor grid has
+// completed and its writes are visible.  Every global-memory access of these
+// kernels comes after that wait, so stream order holds for their data; the
+// wait returns at once when the kernel was launched without the attribute.
+// A dependent grid is launched only after every CTA of its predecessor has
+// signalled (or exited), so a waiting grid never keeps its predecessor's
+// CTAs off the SMs.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_chained(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                           Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int32_t* values,
                                 int n_runs, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, int D, cudaStream_t s);
