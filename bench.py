@@ -590,11 +590,23 @@ def oracle_sample_step(w, dev, layer, task=0):
     return dt, (w.n_aux + 1) / w.n_layers
 
 
+CPU_SAMPLE_S = 10.0  # oracle seconds the cpu_baseline sample aims for (whole layers, at most 30 s)
+
+
 def cpu_baseline(w, dev):
-    dt, units = oracle_sample_step(w, dev, layer=0)
+    """The oracle on the host cores over a bounded sample of the step: whole
+    layers of one fork group, added until about CPU_SAMPLE_S seconds of oracle
+    work."""
+    dt = units = 0.0
+    layers = 0
+    while layers < w.n_layers and dt < CPU_SAMPLE_S:
+        d, u = oracle_sample_step(w, dev, layer=layers)
+        dt += d
+        units += u
+        layers += 1
     return {"value": units / dt, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"1 of {w.n_layers} layers of 1 of {w.n_tasks} fork groups ({w.n_aux + 1} branches, "
-                      f"{w.prefix[0]}-token prefix), float64 numpy; {dt:.1f} s"}
+            "sample": f"{layers} of {w.n_layers} layers of 1 of {w.n_tasks} fork groups ({w.n_aux + 1} branches, "
+                      f"{w.prefix[0]}-token prefix), float64 numpy; {dt:.1f} s of oracle work"}
 
 
 def run_reference(args, rank, ws, local):
