@@ -104,6 +104,22 @@ def _seq_array(seqs):
     return (ctypes.c_int64 * max(1, len(seqs)))(*seqs), len(seqs)
 
 
+class _SeqArrays:
+    """The ctypes handle array of the last branch list passed, reused while the
+    same handles come back (a decode loop passes the same list every step)."""
+
+    def __init__(self):
+        self._key = None
+        self._val = None
+
+    def __call__(self, seqs):
+        key = tuple(seqs)
+        if key != self._key:
+            self._val = _seq_array(key)
+            self._key = key
+        return self._val
+
+
 class Pool:
     """A KV block pool on one GPU (or metadata-only with device=None).
 
@@ -114,6 +130,7 @@ class Pool:
     def __init__(self, n_layers, n_q_heads, n_kv_heads, head_dim, n_blocks, seed=0,
                  max_seqs=64, max_pages=None, max_decode_branches=16, max_splits=16,
                  device="cuda", flags=0):
+        self._seqs = _SeqArrays()
         self.cfg = StConfig(
             n_layers=n_layers, n_q_heads=n_q_heads, n_kv_heads=n_kv_heads, head_dim=head_dim,
             page_size=PAGE, max_seqs=max_seqs,
@@ -156,8 +173,12 @@ class Pool:
     def _stream(self, stream):
         if self.device is None:
             return None
-        import torch
         if stream is None:
+            # the current stream's handle, without building a Stream object
+            import torch
+            raw = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+            if raw is not None:
+                return ctypes.c_void_p(raw(self.device.index))
             stream = torch.cuda.current_stream(self.device)
         return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
 
@@ -204,7 +225,7 @@ class Pool:
     def append_kv(self, branches, k, v, stream=None):
         """k, v: bf16 [L][n_br][n_tok][Hkv][D] (a metadata-only pool takes
         k = v = None and n_tok passed as an int in k's place)."""
-        arr, n = _seq_array(branches)
+        arr, n = self._seqs(branches)
         c = self.cfg
         if self.device is None:
             n_tok = int(k)
@@ -220,7 +241,7 @@ class Pool:
     def decode_attn(self, branches, q, o=None, lse=None, stream=None):
         """q: bf16 [L][n_br][Hq][D] -> (o fp32 [L][n_br][Hq][D], lse fp32 [L][n_br][Hq])."""
         import torch
-        arr, n = _seq_array(branches)
+        arr, n = self._seqs(branches)
         c = self.cfg
         qp = self._dev(q, torch.bfloat16, (c.n_layers, n, c.n_q_heads, c.head_dim), "q")
         if o is None:

@@ -108,6 +108,35 @@ def test_cfg4_long_trajectory_sampled_layers(stlib):
         compare(o[layer], lse[layer], o_ref, l_ref, f"cfg4 layer {layer}")
 
 
+@pytest.mark.parametrize("n_aux", [8, 16])
+def test_cfg4_long_trajectory_wide_sampled_layers(stlib, n_aux):
+    """The long-trajectory workload at full size with 9 branches per group (72
+    stacked rows: one wide tile per group) and 17 (136 rows: two wide subgroups
+    whose second read of each prefix page comes from L2), as `bench.py --n-aux`
+    times it."""
+    from workloads.configs import long_with_branches
+    w = long_with_branches(n_aux)
+    run = _run(w, cache_layers=48)
+    groups = []
+    for t in range(w.n_tasks):
+        m = run.create()
+        _prefix(run, m, w.prefix[t], ("prefix", t))
+        aux = run.fork(m, w.n_aux)
+        br = [m] + aux
+        for b, (rid, s) in enumerate(zip(br, w.suffix[t])):
+            if s:
+                run.append([rid], s, ("suffix", t, b))
+        groups.append(br)
+    rids = [r for g in groups for r in g]
+    run.append(rids, 1, ("step",))
+    q, o, lse = run.decode(rids, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    for layer in (0, w.n_layers - 1):
+        o_ref, l_ref = run.oracle_decode(rids, q, layer)
+        compare(o[layer], lse[layer], o_ref, l_ref, f"{w.name} layer {layer}")
+
+
 def test_cfg5_full_cycle_sampled(stlib):
     w = get(5)
     run = _run(w, cache_layers=32)
