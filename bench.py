@@ -136,16 +136,16 @@ def _kernel_hash():
     return h.hexdigest()[:16]
 
 
-def _ncu_traffic(kernel):
+def _ncu_traffic(kernel, workload):
     """dram bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source."""
+    on the current kernel source and on this workload."""
     try:
         with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
             d = json.load(f)
     except OSError:
         return None
     e = d.get(kernel)
-    if not e or e.get("source_hash") != _kernel_hash():
+    if not e or e.get("source_hash") != _kernel_hash() or e.get("workload") != workload:
         return None
     return e.get("dram_bytes_per_launch")
 
@@ -309,7 +309,7 @@ def run_ours(args, rank, ws, local):
                          "peak": peaks["hbm_gbs"], "peak_source": src, "unit": "GB/s",
                          "frac": achieved / peaks["hbm_gbs"], "frac_of_nominal_8tbs": achieved / 8000.0,
                          "bytes_per_launch": bytes_per_launch, "avg_launch_ms": avg_ms,
-                         "traffic": _ncu_traffic("decode_partial")},
+                         "traffic": _ncu_traffic("decode_partial", w.name)},
             "kernels": {k: {"launches": v["launches"], "ms": v["total_ms"]} for k, v in stats.items()
                         if v["launches"]},
             "gpu_launches": launches,

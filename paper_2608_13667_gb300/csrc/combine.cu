@@ -27,8 +27,35 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
   if (idx >= total) return;
   const int b = (int)((idx / p.Hq) % p.n_br);
   const int ns = n_splits[b];
+  constexpr int kPer = D / 32;
+  constexpr int kBatch = 16;  // partials whose loads are in flight together
   const float* lse_i = p.part_lse + idx * p.max_splits;
+  const float* po = p.part_o + idx * p.max_splits * D + lane * kPer;
+  // this lane's column slice of partial i (zero past the branch's partials)
+  auto load = [&](int i, float* x) {
+    if (i < ns) {
+      if constexpr (kPer == 4) {
+        const float4 v = *reinterpret_cast<const float4*>(po + (int64_t)i * D);
+        x[0] = v.x;
+        x[1] = v.y;
+        x[2] = v.z;
+        x[3] = v.w;
+      } else {
+        const float2 v = *reinterpret_cast<const float2*>(po + (int64_t)i * D);
+        x[0] = v.x;
+        x[1] = v.y;
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) x[e] = 0.f;
+    }
+  };
+  // the first batch of partials is loaded together with the lse values: the
+  // loads do not depend on the weights
   const float li = lane < ns ? lse_i[lane] : -INFINITY;
+  float x[kBatch][kPer];
+#pragma unroll
+  for (int u = 0; u < kBatch; ++u) load(u, x[u]);
   float mx = li;
 #pragma unroll
   for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
@@ -37,42 +64,21 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
 #pragma unroll
   for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
   const float lse = mx + logf(sum);
-  constexpr int kPer = D / 32;
-  constexpr int kBatch = 8;  // partials whose loads are in flight together
   const float inv_sum = 1.f / sum;
   float out[kPer];
 #pragma unroll
   for (int e = 0; e < kPer; ++e) out[e] = 0.f;
-  const float* po = p.part_o + idx * p.max_splits * D + lane * kPer;
   for (int i0 = 0; i0 < ns; i0 += kBatch) {
-    float x[kBatch][kPer];
-    float wv[kBatch];
+    if (i0 > 0) {
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      const int i = i0 + u;
-      wv[u] = __shfl_sync(0xffffffffu, w, i & 31) * inv_sum;
-      if (i < ns) {
-        if constexpr (kPer == 4) {
-          const float4 v = *reinterpret_cast<const float4*>(po + (int64_t)i * D);
-          x[u][0] = v.x;
-          x[u][1] = v.y;
-          x[u][2] = v.z;
-          x[u][3] = v.w;
-        } else {
-          const float2 v = *reinterpret_cast<const float2*>(po + (int64_t)i * D);
-          x[u][0] = v.x;
-          x[u][1] = v.y;
-        }
-      } else {
-        wv[u] = 0.f;
-#pragma unroll
-        for (int e = 0; e < kPer; ++e) x[u][e] = 0.f;
-      }
+      for (int u = 0; u < kBatch; ++u) load(i0 + u, x[u]);
     }
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u)
+    for (int u = 0; u < kBatch; ++u) {
+      const float wv = i0 + u < ns ? __shfl_sync(0xffffffffu, w, (i0 + u) & 31) * inv_sum : 0.f;
 #pragma unroll
-      for (int e = 0; e < kPer; ++e) out[e] += wv[u] * x[u][e];
+      for (int e = 0; e < kPer; ++e) out[e] += wv * x[u][e];
+    }
   }
   float* dst = p.o + idx * D + lane * kPer;
   if (kPer == 4)
