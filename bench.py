@@ -526,6 +526,8 @@ def run_cycle():
     ml = torch.empty((L, w.merge_tokens, w.n_q_heads), dtype=torch.float32, device=dev)
     torch.cuda.synchronize(dev)
     pool.profile_enable(True)
+    t_fork = t_release = 0.0  # host time of the metadata-only calls (no GPU work)
+    n_fork = n_release = 0
     t_all = time.perf_counter()
     for turn in range(w.turns):
         singles = [pool.seq_create() for _ in range(w.singletons)]
@@ -533,16 +535,22 @@ def run_cycle():
             k, v = kv_rows(w, ("single", turn, i), 8 * w.singleton_len, device=dev)
             pool.append_kv(singles[i:i + 8], k.view(L, 8, w.singleton_len, Hkv, D),
                            v.view(L, 8, w.singleton_len, Hkv, D))
+        t0 = time.perf_counter()
         groups = [[m] + pool.fork(m, w.n_aux) for m in mains]
+        t_fork += time.perf_counter() - t0
+        n_fork += len(mains)
         rids = [r for g in groups for r in g] + singles
         for step in range(w.steps):
             pool.append_kv(rids, sk, sv)
             pool.decode_attn(rids, sq, o, lse)
         for m in mains:
             pool.merge(m, mq, mk, mv, mo, ml)
+        t0 = time.perf_counter()
         for g in groups:
             for a in g[1:]:
                 pool.release(a)
+        t_release += time.perf_counter() - t0
+        n_release += sum(len(g) - 1 for g in groups)
         for s_ in singles:
             pool.release(s_)
     torch.cuda.synchronize(dev)
@@ -557,6 +565,8 @@ def run_cycle():
         "branch_steps_per_s": dec["launches"] * n_rows / total,
         "merges": mer["launches"], "merge_ms": mer["total_ms"] / mer["launches"],
         "merge_tflops": mer["flops"] / mer["total_ms"] / 1e9,
+        "fork_us": t_fork / n_fork * 1e6, "fork_note": f"st_fork of {w.n_aux} branches off a main context, host time through the binding",
+        "release_us": t_release / n_release * 1e6, "release_note": "st_release of one branch, host time through the binding",
         "kernels": {k: {"launches": v["launches"], "ms": v["total_ms"]} for k, v in stats.items() if v["launches"]}}))
 
 
