@@ -128,11 +128,20 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def _code_only(src):
+    """C++ source without comments and whitespace (a comment edit is not a
+    kernel change)."""
+    import re
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", " ", src)
+    return re.sub(r"\s+", "", src)
+
+
 def _kernel_hash():
     h = hashlib.sha256()
     for f in ("attend_tc.cu", "ptx.cuh", "kernels.cuh"):
-        with open(os.path.join(ROOT, "paper_2608_13667_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2608_13667_gb300", "csrc", f)) as fh:
+            h.update(_code_only(fh.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -35,12 +35,19 @@
 //   warp 4      loader: page ids from the block table (32 per read, one batch
 //               ahead), one 2 KiB TMA copy per (page, 64-wide half of D, K|V)
 //               into a ring of stages, per-stage mbarriers with byte counts.
+//               Narrow: one ring, a stage's K and V slots freed together after
+//               its P V.  Wide: K and V have their own barriers; a K slot is
+//               freed by the commit after S_j, a V slot after P_j V_j.
 //   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M, N=64 keys)
 //               and O += P V (M, N=D) and commits them to mbarriers.  S is
 //               double-buffered in TMEM: S_{j+1} is issued before P_j V_j when
 //               its data has landed, so the softmax of stage j+1 overlaps the
 //               tensor work of stage j.
 //               A rescale of O first waits for the commit of P_{j-1} V_{j-1}.
+//
+// The kernel is launched as a programmatic dependent of the append before it
+// in the stream: the TMEM allocation comes before griddepcontrol.wait, every
+// global-memory access after it.
 //
 // Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
 //   Q  [D/64][rows][64]       K-major A (SBO 1024)
