@@ -194,8 +194,10 @@ __global__ void __launch_bounds__(kThreads, 2)
       prefetch_tensormap(&vmap);
     }
     // a page is streamed once, unless a sibling item (the group's other
-    // subgroup, scheduled next to this one) reads it too: then keep it in L2
-    const uint64_t policy = (item.flags & kItemReread) ? l2_policy_evict_normal() : l2_policy_evict_first();
+    // subgroup, scheduled next to this one) reads it too, or the whole launch
+    // fits in L2 (one agent's step, read again by the next step): then keep it
+    const uint64_t policy =
+        (p.keep_l2 || (item.flags & kItemReread)) ? l2_policy_evict_normal() : l2_policy_evict_first();
     const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;

@@ -98,6 +98,7 @@ struct AttnParams {
   int32_t slot, L0, T;     // merge only: main's slot, length before the append, thought rows
   int32_t hold_loads;      // test hook (ST_FLAG_HOLD_LOADS): the loader issues nothing
   int32_t item_base;       // decode: CTA x reads item item_base + x
+  int32_t keep_l2;         // decode: the launch's pages fit in L2; load them evict-normal so they stay
   const MergeItem* mitems; // batched merge: CTA x takes mitems[x] (slot, L0, T above unused)
 };
 

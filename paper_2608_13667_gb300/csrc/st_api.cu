@@ -131,6 +131,7 @@ struct st_pool {
   float* d_part_lse = nullptr;
   CUtensorMap kmap{}, vmap{};
   int sms = 0, decode_ctas_per_sm = 0;
+  int64_t l2_bytes = 0;
   // staging ring
   uint8_t* h_stage = nullptr;
   cudaEvent_t stage_ev[kStageSlots] = {};
@@ -491,6 +492,11 @@ ST_API st_status st_pool_create(const st_config* cfg, void* k_pool, void* v_pool
   if (cudaMemset(P->ws, 0, P->lay.staging) != cudaSuccess) return bail(ST_ERR_CUDA);
   if (cudaDeviceGetAttribute(&P->sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
     return bail(ST_ERR_CUDA);
+  {
+    int l2 = 0;
+    if (cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, device) != cudaSuccess) return bail(ST_ERR_CUDA);
+    P->l2_bytes = l2;
+  }
   P->decode_ctas_per_sm = decode_tc_ctas_per_sm(cfg->head_dim);
   if (P->decode_ctas_per_sm < 1) return bail(ST_ERR_CUDA);
   if (cudaHostAlloc(reinterpret_cast<void**>(&P->h_stage), (size_t)kStageSlots * kStageSlotBytes,
@@ -857,6 +863,9 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.max_pages = c.max_pages;
   ap.max_splits = c.max_splits;
   ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
+  // a launch whose pages take less than half of L2 is one agent's step or a
+  // few: the next step reads the same pages, so they stay in L2
+  ap.keep_l2 = bytes < 0.5 * (double)P->l2_bytes ? 1 : 0;
   const int n_items = (int)items.size();
   int n_narrow = 0;
   while (n_narrow < n_items && !(items[n_narrow].flags & kItemWide)) ++n_narrow;
