@@ -228,17 +228,19 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       return np;
     };
-    // wide: np pages of one operand into a slot, completing on bar (lane 0 issues)
+    // wide: np pages of one operand into a slot, completing on bar, one copy
+    // per lane (lane = D/64 q + h), after lane 0's expect-tx
     const uint32_t page_bytes = (uint32_t)(C::kHalves * kPageTokens * 128);
     auto issue = [&](const CUtensorMap* map, uint8_t* dst, uint64_t* bar, const int* c3, int np) {
-      if (lane != 0) return;
+      __syncwarp();
+      const int q = lane / C::kHalves, h = lane % C::kHalves;
+      int cq = c3[0];
 #pragma unroll
-      for (int q = 0; q < C::kPagesPerStage; ++q)
-#pragma unroll
-        for (int h = 0; h < C::kHalves; ++h)
-          if (q < np)
-            tma_load_4d(dst + h * C::kKVHalfBytes + q * kPageTokens * 128, map, bar, 0, h, kvh * kPageTokens,
-                        c3[q], policy);
+      for (int i = 1; i < C::kPagesPerStage; ++i)
+        if (q == i) cq = c3[i];
+      if (lane < C::kHalves * np)
+        tma_load_4d(dst + h * C::kKVHalfBytes + q * kPageTokens * 128, map, bar, 0, h, kvh * kPageTokens, cq,
+                    policy);
     };
     int jk = 0, jv = 0;  // stages whose K and V copies have been issued
     bool ok = true;
@@ -272,27 +274,22 @@ __global__ void __launch_bounds__(kThreads, 2)
           nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
         }
         const int np = min(C::kPagesPerStage, n_pages - page0);
-        int blk[C::kPagesPerStage];
-#pragma unroll
-        for (int q = 0; q < C::kPagesPerStage; ++q)
-          blk[q] = __shfl_sync(0xffffffffu, cur, (page0 - base_id + q) & 31);
-        if (lane == 0) {
-          mbar_arrive_expect_tx(&full[s], 2 * np * page_bytes);
-          for (int q = 0; q < np; ++q) {
-            int b = blk[q];
-            if ((uint64_t)b >= (uint64_t)p.n_blocks) {
-              atomicCAS(p.status, 0, kDevBadIndex);
-              b = 0;
-            }
-            const int c3 = layer * (int)p.n_blocks + b;
-#pragma unroll
-            for (int h = 0; h < C::kHalves; ++h) {
-              tma_load_4d(kst + h * C::kKVHalfBytes + q * kPageTokens * 128, &kmap, &full[s], 0, h,
-                          kvh * kPageTokens, c3, policy);
-              tma_load_4d(vst + h * C::kKVHalfBytes + q * kPageTokens * 128, &vmap, &full[s], 0, h,
-                          kvh * kPageTokens, c3, policy);
-            }
+        if (lane == 0) mbar_arrive_expect_tx(&full[s], 2 * np * page_bytes);
+        __syncwarp();
+        // one copy per lane (lane = 2 D/64 q + (V ? D/64 : 0) + h): a single
+        // thread issuing them one after another is what limits the stage rate
+        constexpr int kPerPage = 2 * C::kHalves;
+        const int q = lane / kPerPage, r = lane % kPerPage;
+        const int h = r % C::kHalves;
+        const bool is_v = r >= C::kHalves;
+        int b = __shfl_sync(0xffffffffu, cur, (page0 - base_id + (q < C::kPagesPerStage ? q : 0)) & 31);
+        if (lane < kPerPage * np) {
+          if ((uint64_t)b >= (uint64_t)p.n_blocks) {
+            atomicCAS(p.status, 0, kDevBadIndex);
+            b = 0;
           }
+          tma_load_4d((is_v ? vst : kst) + h * C::kKVHalfBytes + q * kPageTokens * 128, is_v ? &vmap : &kmap,
+                      &full[s], 0, h, kvh * kPageTokens, layer * (int)p.n_blocks + b, policy);
         }
       }
     }
