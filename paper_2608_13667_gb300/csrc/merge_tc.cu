@@ -203,24 +203,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
       }
       const int np = min(kPagesPerStage, n_pages - page0);
-      int blk[kPagesPerStage];
-#pragma unroll
-      for (int q = 0; q < kPagesPerStage; ++q) blk[q] = __shfl_sync(0xffffffffu, cur, (page0 - base_id + q) & 31);
-      if (lane == 0) {
-        uint8_t* dst = ring + s * C::kSlotBytes;
-        mbar_arrive_expect_tx(&full[s], (uint32_t)(np * C::kHalves * kPageTokens * 128));
-        for (int q = 0; q < np; ++q) {
-          int b = blk[q];
-          if ((uint64_t)b >= (uint64_t)p.n_blocks) {
-            atomicCAS(p.status, 0, kDevBadIndex);
-            b = 0;
-          }
-          const int c3 = layer * (int)p.n_blocks + b;
-#pragma unroll
-          for (int h = 0; h < C::kHalves; ++h)
-            tma_load_4d(dst + h * C::kKVHalfBytes + q * kPageTokens * 128, map, &full[s], 0, h,
-                        kvh * kPageTokens, c3, policy);
+      uint8_t* dst = ring + s * C::kSlotBytes;
+      if (lane == 0) mbar_arrive_expect_tx(&full[s], (uint32_t)(np * C::kHalves * kPageTokens * 128));
+      __syncwarp();
+      // one copy per lane (lane = D/64 q + h)
+      const int q = lane / C::kHalves, h = lane % C::kHalves;
+      int b = __shfl_sync(0xffffffffu, cur, (page0 - base_id + (q < kPagesPerStage ? q : 0)) & 31);
+      if (lane < C::kHalves * np) {
+        if ((uint64_t)b >= (uint64_t)p.n_blocks) {
+          atomicCAS(p.status, 0, kDevBadIndex);
+          b = 0;
         }
+        tma_load_4d(dst + h * C::kKVHalfBytes + q * kPageTokens * 128, map, &full[s], 0, h, kvh * kPageTokens,
+                    layer * (int)p.n_blocks + b, policy);
       }
     }
     if (!ok && lane == 0) {
