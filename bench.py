@@ -467,6 +467,56 @@ def run_profile_wide():
                       "decode_gbs": d["bytes"] / d["total_ms"] / 1e6}))
 
 
+def run_harvest():
+    """The thought harvest (st_harvest) on token ids: 4 branches x 512 generated
+    tokens (one turn's aux branches at the cycle's 512 steps) and 32 x 2048.
+    Seeded streams with open/close tags at 6% / 8% of positions.  Prints the
+    device time per call (200 calls back to back, CUDA events) and the latency
+    of one call through the binding, including the read-back of the count."""
+    import ctypes
+    import numpy as np
+    import torch
+    import paper_2608_13667_gb300 as st
+    st.build()
+    L = st.lib()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    res = {}
+    for n_br, stride in ((4, 512), (32, 2048)):
+        rng = np.random.default_rng(n_br)
+        s = rng.integers(100, 5000, size=(n_br, stride)).astype(np.int32)
+        r = rng.random((n_br, stride))
+        s[r < 0.06] = 7
+        s[(r >= 0.06) & (r < 0.14)] = 8
+        ds = torch.from_numpy(s).to(dev)
+        dl = torch.full((n_br,), stride, dtype=torch.int32, device=dev)
+        ids = torch.empty(n_br * stride, dtype=torch.int32, device=dev)
+        src = torch.empty_like(ids)
+        atoms = torch.empty(n_br, dtype=torch.int32, device=dev)
+        count = torch.empty(1, dtype=torch.int32, device=dev)
+        args = (ctypes.c_void_p(ds.data_ptr()), stride, ctypes.c_void_p(dl.data_ptr()), n_br, 7, 8, 5,
+                ctypes.c_void_p(ids.data_ptr()), ctypes.c_void_p(src.data_ptr()), ctypes.c_void_p(atoms.data_ptr()),
+                ctypes.c_void_p(count.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+        for _ in range(10):
+            assert L.st_harvest(*args) == 0
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n = 200
+        e0.record(stream)
+        for _ in range(n):
+            L.st_harvest(*args)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        dev_us = e0.elapsed_time(e1) / n * 1e3
+        t0 = time.perf_counter()
+        for _ in range(20):
+            st.st_harvest(ds, dl, 7, 8, 5)
+        lat_us = (time.perf_counter() - t0) / 20 * 1e6
+        res[f"{n_br}x{stride}"] = {"device_us_per_call": dev_us, "latency_us_with_readback": lat_us,
+                                   "harvested_tokens": int(count.item())}
+    print(json.dumps({"workload": "thought harvest on token ids", **res}))
+
+
 def run_prefill_batch():
     """Batched prefill on the batched-serving shape (1 layer, 32/8 heads, D 128):
     16 agents with contexts of 4096-32768 tokens each receive an observation of
@@ -703,6 +753,8 @@ def main():
                     help="run the small decode + merge case used for ncu captures and exit")
     ap.add_argument("--profile-wide", action="store_true",
                     help="run the small 9-branch decode case (wide tile) used for ncu captures and exit")
+    ap.add_argument("--harvest", action="store_true",
+                    help="time the thought harvest (st_harvest) and exit")
     ap.add_argument("--prefill-batch", action="store_true",
                     help="time one batched prefill of 16 agents against one merge per agent and exit")
     ap.add_argument("--profile-merge", action="store_true",
@@ -718,6 +770,9 @@ def main():
         return
     if args.prefill_batch:
         run_prefill_batch()
+        return
+    if args.harvest:
+        run_harvest()
         return
     if args.profile_wide:
         run_profile_wide()
