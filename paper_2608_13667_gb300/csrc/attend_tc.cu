@@ -34,7 +34,8 @@
 //               split-KV partial with its log-sum-exp.
 //   warp 4      loader: page ids from the block table (32 per read, one batch
 //               ahead), one 2 KiB TMA copy per (page, 64-wide half of D, K|V)
-//               into a ring of stages, per-stage mbarriers with byte counts.
+//               into a ring of stages, per-stage mbarriers with byte counts;
+//               a stage's copies are issued by the warp's lanes together.
 //               Narrow: one ring, a stage's K and V slots freed together after
 //               its P V.  Wide: K and V have their own barriers; a K slot is
 //               freed by the commit after S_j, a V slot after P_j V_j.
