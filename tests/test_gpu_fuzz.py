@@ -71,3 +71,37 @@ def test_random_fork_groups(stlib, seed):
         off += n
     run.pool.sync()
     run.check_tables()
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_large_fork_groups(stlib, seed):
+    """Large fork groups: 7 to 21 branches at G = 4 or 8 (28 to 168 stacked
+    rows: wide tiles, and balanced wide subgroups beyond 128 rows), prefixes
+    of up to 6000 tokens with random fork points, ragged suffixes."""
+    rng = np.random.default_rng(5000 + seed)
+    D = int(rng.choice([64, 128]))
+    Hkv = int(rng.choice([1, 2, 4]))
+    G = int(rng.choice([4, 8]))
+    w = Workload(name=f"fuzz_large{seed}", n_layers=1, n_q_heads=Hkv * G, n_kv_heads=Hkv, head_dim=D,
+                 n_blocks=2048, seed=seed)
+    run = Run(w, max_seqs=48, max_decode_branches=48, max_splits=int(rng.choice([4, 16, 32])))
+    rids = []
+    for g in range(int(rng.integers(1, 3))):
+        m = run.create()
+        run.append([m], int(rng.integers(200, 6000)), ("p", g))
+        n_aux = int(rng.integers(6, 21))
+        point = run.ref.seqs[m].length if rng.random() < 0.5 else int(rng.integers(0, run.ref.seqs[m].length + 1))
+        kids = run.fork_at(m, point, n_aux)
+        for b, r in enumerate([m] + kids):
+            s = int(rng.integers(0, 90))
+            if s:
+                run.append([r], s, ("s", g, b))
+        rids += [r for r in [m] + kids if run.ref.seqs[r].length > 0]
+    rng.shuffle(rids)
+    for step in range(2):
+        run.append(rids, 1, ("step", step))
+        q, o, lse = run.decode(rids, ("q", step))
+        o_ref, l_ref = run.oracle_decode(rids, q, 0)
+        compare(o[0], lse[0], o_ref, l_ref, f"seed {seed} step {step}")
+    run.pool.sync()
+    run.check_tables()
