@@ -330,7 +330,7 @@ def run_ours(args, rank, ws, local):
     if rank == 0:
         peaks, src = _peaks()
         dec = stats["decode_partial"]
-        launches = sum(v["launches"] for v in stats.values())
+        launches = sum(v["kernels"] for v in stats.values())  # device kernels, not calls
         avg_ms = dec["total_ms"] / max(1, dec["launches"])
         bytes_per_launch = dec["bytes"] / max(1, dec["launches"])
         achieved = bytes_per_launch / (avg_ms * 1e-3) / 1e9
@@ -352,8 +352,8 @@ def run_ours(args, rank, ws, local):
                          "frac": achieved / peaks["hbm_gbs"], "frac_of_nominal_8tbs": achieved / 8000.0,
                          "bytes_per_launch": bytes_per_launch, "avg_launch_ms": avg_ms,
                          "traffic": _ncu_traffic("decode_partial", w.name)},
-            "kernels": {k: {"launches": v["launches"], "ms": v["total_ms"]} for k, v in stats.items()
-                        if v["launches"]},
+            "kernels": {k: {"launches": v["launches"], "device_kernels": v["kernels"], "ms": v["total_ms"]}
+                        for k, v in stats.items() if v["launches"]},
             "gpu_launches": launches,
             "clocks": clk,
             "e2e": {"value": ws * n_br * e2e_steps / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,

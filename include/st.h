@@ -234,6 +234,8 @@ typedef struct {
   double total_ms;     /* summed event time (0 when timing was off) */
   double bytes;        /* algorithmic bytes the launches had to move */
   double flops;        /* algorithmic floating-point operations */
+  int64_t kernels;     /* device kernels launched (a decode call with both tile
+                          shapes launches two per call) */
 } st_kernel_stat;
 ST_API st_status st_profile_enable(st_pool* pool, int enable);
 ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, int* n);

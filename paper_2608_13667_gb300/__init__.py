@@ -50,6 +50,7 @@ class StKernelStat(ctypes.Structure):
         ("total_ms", ctypes.c_double),
         ("bytes", ctypes.c_double),
         ("flops", ctypes.c_double),
+        ("kernels", ctypes.c_int64),
     ]
 
 
@@ -340,7 +341,8 @@ class Pool:
         n = ctypes.c_int()
         self._check(lib().st_profile_read(self._h, buf, 16, ctypes.byref(n)), "st_profile_read")
         return {buf[i].name.decode(): dict(launches=buf[i].launches, total_ms=buf[i].total_ms,
-                                           bytes=buf[i].bytes, flops=buf[i].flops) for i in range(n.value)}
+                                           bytes=buf[i].bytes, flops=buf[i].flops, kernels=buf[i].kernels)
+                for i in range(n.value)}
 
 
 # C-named entry points (argument marshalling only)

@@ -88,7 +88,8 @@ WorkspaceLayout layout_for(const st_config* c) {
 }
 
 struct KStat {
-  int64_t launches = 0;
+  int64_t launches = 0;  // calls of this kind
+  int64_t kernels = 0;   // device kernels they launched
   double ms = 0, bytes = 0, flops = 0;
 };
 
@@ -206,10 +207,12 @@ cudaEvent_t take_event(st_pool* P) {
   return e;
 }
 
-// Launch wrapper: counts the launch, adds its algorithmic bytes/flops, and
-// brackets it with events when timing is on.
+// Launch wrapper: counts the launch (and the n_kernels device kernels it
+// makes), adds its algorithmic bytes/flops, and brackets it with events when
+// timing is on.
 template <class F>
-st_status run_kernel(st_pool* P, int kid, double bytes, double flops, cudaStream_t s, F&& launch) {
+st_status run_kernel(st_pool* P, int kid, double bytes, double flops, cudaStream_t s, F&& launch,
+                     int n_kernels = 1) {
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (P->timing) {
     e0 = take_event(P);
@@ -225,6 +228,7 @@ st_status run_kernel(st_pool* P, int kid, double bytes, double flops, cudaStream
   }
   KStat& k = P->stats[kid];
   k.launches += 1;
+  k.kernels += n_kernels;
   k.bytes += bytes;
   k.flops += flops;
   return ST_OK;
@@ -876,7 +880,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     AttnParams aw = ap;
     aw.item_base = n_narrow;
     return launch_decode_tc(P->kmap, P->vmap, aw, ip, n_items - n_narrow, c.head_dim, true, s);
-  });
+  }, (n_narrow > 0 ? 1 : 0) + (n_items > n_narrow ? 1 : 0));
   if (st != ST_OK) return st;
 
   CombineParams cp{};
@@ -1110,6 +1114,7 @@ ST_API st_status st_profile_read(st_pool* P, st_kernel_stat* out, int cap, int* 
       out[k].total_ms = P->stats[i].ms;
       out[k].bytes = P->stats[i].bytes;
       out[k].flops = P->stats[i].flops;
+      out[k].kernels = P->stats[i].kernels;
       ++k;
     }
     P->stats[i] = KStat{};

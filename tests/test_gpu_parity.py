@@ -405,3 +405,25 @@ def test_fork_point_variants(stlib, variant):
                 compare(o[layer], lse[layer], o_ref, l_ref, f"{variant} step {step} layer {layer}")
     run.pool.sync()
     run.check_tables()
+
+
+def test_profile_counts_device_kernels(stlib):
+    """A decode call whose fork group needs the wide tile (9 branches x G = 8 =
+    72 stacked rows) while each branch's own pages take narrow tiles launches
+    two decode kernels; the profile counts calls and kernels apart."""
+    w = Workload(name="kernel_count", n_layers=1, n_q_heads=8, n_kv_heads=1, head_dim=64, n_blocks=256, seed=0)
+    run = Run(w, max_seqs=16, max_decode_branches=16, max_splits=8)
+    m = run.create()
+    run.append([m], 256, ("p",))
+    rids = [m] + run.fork(m, 8)
+    for b, r in enumerate(rids):
+        run.append([r], 20, ("s", b))
+    run.pool.profile_read()
+    q, o, lse = run.decode(rids, ("q",))
+    st = run.pool.profile_read()["decode_partial"]
+    assert (st["launches"], st["kernels"]) == (1, 2)
+    o_ref, l_ref = run.oracle_decode(rids, q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "wide + narrow")
+    q, o, lse = run.decode(rids[:2], ("q2",))  # 16 rows: narrow tiles only
+    st = run.pool.profile_read()["decode_partial"]
+    assert (st["launches"], st["kernels"]) == (1, 1)
