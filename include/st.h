@@ -153,6 +153,28 @@ ST_API st_status st_append_kv(st_pool* pool, const st_seq* br, int n_br, int n_t
 ST_API st_status st_decode_attn(st_pool* pool, const st_seq* br, int n_br, const void* q, float* o,
                                 float* lse, void* stream);
 
+/* The work decomposition st_decode_attn would use for these branches, without
+ * launching anything (host only; also on a metadata-only pool, which plans for
+ * 152 SMs with two decode CTAs each).  One item is a run of pages of one
+ * block table read for a set of branches, one CTA per KV head and layer:
+ * items:    int32 [item_cap][8] rows {owner, page_begin, n_pages, n_tokens,
+ *           member_base, n_members, split, flags}: owner is the index in br
+ *           of the branch whose block table the run is read from, pages
+ *           [page_begin, page_begin + n_pages) of it, n_tokens valid keys,
+ *           members[member_base .. + n_members) the branches (indices in br)
+ *           whose query rows are stacked on it, split the partial slot it
+ *           writes for each of them; flags bit 0: a sibling item of the same
+ *           fork family reads the same pages (kept in L2), bit 1: the wide
+ *           (M = 128) tile.  Narrow items come first.
+ * members:  int32 [member_cap]
+ * n_splits: int32 [n_br], partial results per branch (each split index
+ *           0 .. n_splits - 1 is written by exactly one item)
+ * *n_items and *n_members receive the sizes the plan needs; ST_ERR_INVALID
+ * (nothing written) when they exceed item_cap or member_cap. */
+ST_API st_status st_decode_plan(st_pool* pool, const st_seq* br, int n_br, int32_t* items, int item_cap,
+                                int32_t* members, int member_cap, int32_t* n_splits, int* n_items,
+                                int* n_members);
+
 /* Merge (Section 3.5): append the n_tok harvested thought rows to `main`
  * (same rules as st_append_kv) and run their causal prefill: thought row i
  * attends over main's rows [0, L0 + i] inclusive, L0 = main's length before

@@ -78,6 +78,7 @@ def lib():
         "st_fork_at": (I, [P, I64, I64, I, i64p]),
         "st_append_kv": (I, [P, i64p, I, I, VP, VP, VP]),
         "st_decode_attn": (I, [P, i64p, I, VP, VP, VP, VP]),
+        "st_decode_plan": (I, [P, i64p, I, i32p, I, i32p, I, i32p, ctypes.POINTER(I), ctypes.POINTER(I)]),
         "st_merge": (I, [P, I64, I, VP, VP, VP, VP, VP, VP]),
         "st_prefill_batch": (I, [P, i64p, I, i32p, VP, VP, VP, VP, VP, VP]),
         "st_release": (I, [P, I64]),
@@ -253,6 +254,25 @@ class Pool:
         lp = self._dev(lse, torch.float32, (c.n_layers, n, c.n_q_heads), "lse")
         self._check(lib().st_decode_attn(self._h, arr, n, qp, op, lp, self._stream(stream)), "st_decode_attn")
         return o, lse
+
+    def decode_plan(self, branches):
+        """The work decomposition st_decode_attn uses for these branches (host
+        only, also on a metadata-only pool): (items, members, n_splits), items a
+        list of dicts with the fields of include/st.h."""
+        arr, n = _seq_array(branches)
+        L = lib()
+        ni, nm = ctypes.c_int(), ctypes.c_int()
+        st = L.st_decode_plan(self._h, arr, n, None, 0, None, 0, None, ctypes.byref(ni), ctypes.byref(nm))
+        if st != ST_OK and ni.value == 0:  # a rejected call (a plan has at least one item), not a size query
+            self._check(st, "st_decode_plan")
+        items = (ctypes.c_int32 * (8 * max(1, ni.value)))()
+        members = (ctypes.c_int32 * max(1, nm.value))()
+        n_splits = (ctypes.c_int32 * n)()
+        self._check(L.st_decode_plan(self._h, arr, n, items, ni.value, members, nm.value, n_splits, ctypes.byref(ni),
+                                     ctypes.byref(nm)), "st_decode_plan")
+        names = ("owner", "page_begin", "n_pages", "n_tokens", "member_base", "n_members", "split", "flags")
+        rows = [dict(zip(names, items[8 * k:8 * k + 8])) for k in range(ni.value)]
+        return rows, list(members[:nm.value]), list(n_splits)
 
     def merge(self, main, q, k, v, o=None, lse=None, stream=None):
         """q: bf16 [L][T][Hq][D]; k, v: bf16 [L][T][Hkv][D] -> (o [L][T][Hq][D], lse [L][T][Hq])."""

@@ -629,29 +629,29 @@ ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok,
   return do_append(P, slots.data(), n_br, n_tok, k, v, static_cast<cudaStream_t>(stream));
 }
 
-ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const void* q, float* o,
-                                float* lse, void* stream) {
-  NvtxRange range_("st_decode_attn");
-  if (!P) return ST_ERR_INVALID;
-  if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
-  if (n_br < 1 || !br) return fail(P, ST_ERR_INVALID, "need at least one branch");
-  if (n_br > P->cfg.max_decode_branches)
-    return fail(P, ST_ERR_INVALID, "n_br %d > max_decode_branches %d", n_br, P->cfg.max_decode_branches);
-  if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
-    return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
+namespace {
+
+// The decode work decomposition of one st_decode_attn call (host only; the
+// same plan st_decode_plan reports).  Branches are grouped by fork family and
+// the full pages every member of a group holds (the longest common prefix of
+// their block tables) are read once for all of them; each branch's own pages
+// are read for it alone.  Runs of pages are sized to the SM count (about 32
+// waves of two CTAs per SM, at least 16 pages), the tile shape follows the
+// stacked rows (narrow up to 48, wide up to 128, balanced wide subgroups
+// beyond), and the items come out narrow first, longest first.
+struct DecodePlan {
+  std::vector<AttnItem> items;
+  std::vector<int32_t> members;   // the call's branch index of each item's members
+  std::vector<int32_t> n_splits;  // partials per branch
+  double bytes = 0, flops = 0;    // algorithmic, whole launch (KV pages, Q, partials)
+  double part_bytes = 0;          // the partials alone (written here, read by the combine)
+};
+
+void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   BlockPool& bp = *P->pool;
   const st_config& c = P->cfg;
   const int G = c.n_q_heads / c.n_kv_heads;
-  DeviceGuard guard(P->device);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  std::vector<int> slots(n_br);
-  for (int i = 0; i < n_br; ++i) {
-    if (!decode_handle(P, br[i], &slots[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
-    if (bp.slot(slots[i]).len < 1) return fail(P, ST_ERR_INVALID, "decode over an empty sequence");
-    for (int j = 0; j < i; ++j)
-      if (slots[j] == slots[i]) return fail(P, ST_ERR_INVALID, "sequence listed twice");
-  }
-
+  const int n_br = (int)slots.size();
   // ---- group by fork family, find the shared full pages --------------------
   std::vector<int32_t> shared(n_br, 0);   // pages of branch i read through its group
   struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split, wide; };
@@ -716,7 +716,8 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     total_pages += own_pages[i];
   }
   const int64_t units = total_pages * c.n_kv_heads * c.n_layers;
-  const int64_t slots_per_wave = (int64_t)P->sms * P->decode_ctas_per_sm;
+  // a metadata-only pool has no device: it plans for a GB300 (152 SMs, two decode CTAs each)
+  const int64_t slots_per_wave = (int64_t)(P->sms > 0 ? P->sms : 152) * (P->decode_ctas_per_sm > 0 ? P->decode_ctas_per_sm : 2);
   const int64_t target_ctas = 32 * slots_per_wave;
   int64_t chunk = (units + target_ctas - 1) / target_ctas;
   chunk = std::max<int64_t>(16, (chunk + 3) / 4 * 4);
@@ -753,9 +754,6 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
       }
     }
   }
-
-  st_status st = flush_tables(P, s);
-  if (st != ST_OK) return st;
 
   std::vector<AttnItem> items;
   std::vector<int32_t> item_family;  // fork family of a subgroup's item, for scheduling siblings together
@@ -821,6 +819,54 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   part_rows *= (double)c.n_kv_heads * c.n_layers;
   const double part_bytes = part_rows * (c.head_dim + 1) * 4;
   bytes += q_bytes + part_bytes;
+  out->items = std::move(items);
+  out->members = std::move(members);
+  out->n_splits = std::move(n_splits);
+  out->bytes = bytes;
+  out->flops = flops;
+  out->part_bytes = part_bytes;
+}
+
+// The call's branches as pool slots: live, non-empty, each listed once.
+st_status decode_slots(st_pool* P, const st_seq* br, int n_br, std::vector<int>* slots) {
+  if (n_br < 1 || !br) return fail(P, ST_ERR_INVALID, "need at least one branch");
+  if (n_br > P->cfg.max_decode_branches)
+    return fail(P, ST_ERR_INVALID, "n_br %d > max_decode_branches %d", n_br, P->cfg.max_decode_branches);
+  slots->assign(n_br, 0);
+  for (int i = 0; i < n_br; ++i) {
+    if (!decode_handle(P, br[i], &(*slots)[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
+    if (P->pool->slot((*slots)[i]).len < 1) return fail(P, ST_ERR_INVALID, "decode over an empty sequence");
+    for (int j = 0; j < i; ++j)
+      if ((*slots)[j] == (*slots)[i]) return fail(P, ST_ERR_INVALID, "sequence listed twice");
+  }
+  return ST_OK;
+}
+
+}  // namespace
+
+ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const void* q, float* o,
+                                float* lse, void* stream) {
+  NvtxRange range_("st_decode_attn");
+  if (!P) return ST_ERR_INVALID;
+  if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
+  if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
+    return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
+  std::vector<int> slots;
+  st_status vs = decode_slots(P, br, n_br, &slots);
+  if (vs != ST_OK) return vs;
+  const st_config& c = P->cfg;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  DeviceGuard guard(P->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  DecodePlan dp;
+  plan_decode(P, slots, &dp);
+  st_status st = flush_tables(P, s);
+  if (st != ST_OK) return st;
+  const std::vector<AttnItem>& items = dp.items;
+  const std::vector<int32_t>& members = dp.members;
+  const std::vector<int32_t>& n_splits = dp.n_splits;
+  const double bytes = dp.bytes, flops = dp.flops, part_bytes = dp.part_bytes;
 
   // small plans travel in the kernel parameters; larger ones through staging
   const bool inline_plan = items.size() <= (size_t)kInlineItems && members.size() <= (size_t)kInlineMembers &&
@@ -898,6 +944,39 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
                   [&] { return launch_combine(cp, inline_plan ? &inl : nullptr, c.head_dim, s); });
   if (st != ST_OK) return st;
   return inline_plan ? ST_OK : retire_plan(P, ps, s);
+}
+
+ST_API st_status st_decode_plan(st_pool* P, const st_seq* br, int n_br, int32_t* items, int item_cap,
+                                int32_t* members, int member_cap, int32_t* n_splits, int* n_items,
+                                int* n_members) {
+  if (!P) return ST_ERR_INVALID;
+  std::vector<int> slots;
+  st_status vs = decode_slots(P, br, n_br, &slots);
+  if (vs != ST_OK) return vs;
+  DecodePlan dp;
+  plan_decode(P, slots, &dp);
+  if (n_items) *n_items = (int)dp.items.size();
+  if (n_members) *n_members = (int)dp.members.size();
+  if (!items || !members || !n_splits || (int)dp.items.size() > item_cap || (int)dp.members.size() > member_cap)
+    return fail(P, ST_ERR_INVALID, "the plan needs %d items and %d members", (int)dp.items.size(),
+                (int)dp.members.size());
+  for (size_t k = 0; k < dp.items.size(); ++k) {
+    const AttnItem& a = dp.items[k];
+    int owner = 0;
+    while (slots[owner] != a.slot) ++owner;  // every slot of the plan is one of the call's branches
+    int32_t* row = items + 8 * k;
+    row[0] = owner;
+    row[1] = a.page_begin;
+    row[2] = a.n_pages;
+    row[3] = a.n_tokens;
+    row[4] = a.member_base;
+    row[5] = a.n_members;
+    row[6] = a.split;
+    row[7] = a.flags;
+  }
+  std::memcpy(members, dp.members.data(), dp.members.size() * sizeof(int32_t));
+  std::memcpy(n_splits, dp.n_splits.data(), (size_t)n_br * sizeof(int32_t));
+  return ST_OK;
 }
 
 ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, const void* k,
