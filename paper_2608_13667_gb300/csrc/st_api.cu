@@ -1080,6 +1080,12 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
     keys += (double)counts[i] * L0[i] + (double)counts[i] * (counts[i] + 1) / 2;
     q_row0 += counts[i];
   }
+  // longest first (an item's work grows with the keys its rows see, L0 plus
+  // its first token), so that the launch ends on short items, not on the
+  // last tiles of a long context
+  std::stable_sort(items.begin(), items.end(), [&](const MergeItem& x, const MergeItem& y) {
+    return (int64_t)x.L0 + x.row_base / G > (int64_t)y.L0 + y.row_base / G;
+  });
   io_bytes = (double)c.n_layers * R * c.n_q_heads * (c.head_dim * 2 + c.head_dim * 4 + 4);
   const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
   Plan plan;
