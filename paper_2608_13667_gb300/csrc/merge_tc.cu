@@ -127,8 +127,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int layer = blockIdx.z;
   const int G = p.G;
 
-  // one merge: its row tiles in blockIdx.x order; a batch: one work item per CTA
-  int slot = p.slot, L0 = p.L0, T = p.T, q_row0 = 0, row_base = blockIdx.x * 2 * kTileRows;
+  // one merge: its row tiles, the last ones (most keys) first; a batch: one
+  // work item per CTA (the host orders those longest first)
+  int slot = p.slot, L0 = p.L0, T = p.T, q_row0 = 0, row_base = (gridDim.x - 1 - blockIdx.x) * 2 * kTileRows;
   if (p.mitems) {
     const MergeItem mi = p.mitems[blockIdx.x];
     slot = mi.slot;
