@@ -635,7 +635,7 @@ namespace {
 // same plan st_decode_plan reports).  Branches are grouped by fork family and
 // the full pages every member of a group holds (the longest common prefix of
 // their block tables) are read once for all of them; each branch's own pages
-// are read for it alone.  Runs of pages are sized to the SM count (about 32
+// are read for it alone.  Runs of pages are sized to the SM count (about 64
 // waves of two CTAs per SM, at least 16 pages), the tile shape follows the
 // stacked rows (narrow up to 48, wide up to 128, balanced wide subgroups
 // beyond), and the items come out narrow first, longest first.
@@ -718,7 +718,7 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   const int64_t units = total_pages * c.n_kv_heads * c.n_layers;
   // a metadata-only pool has no device: it plans for a GB300 (152 SMs, two decode CTAs each)
   const int64_t slots_per_wave = (int64_t)(P->sms > 0 ? P->sms : 152) * (P->decode_ctas_per_sm > 0 ? P->decode_ctas_per_sm : 2);
-  const int64_t target_ctas = 32 * slots_per_wave;
+  const int64_t target_ctas = 64 * slots_per_wave;
   int64_t chunk = (units + target_ctas - 1) / target_ctas;
   chunk = std::max<int64_t>(16, (chunk + 3) / 4 * 4);
   // Many short runs: each CTA pays a fixed cost (barriers, TMEM, its Q rows,
