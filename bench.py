@@ -467,6 +467,87 @@ def run_profile_wide():
                       "decode_gbs": d["bytes"] / d["total_ms"] / 1e6}))
 
 
+def run_turn():
+    """One agent turn at the paper's shape, phase by phase: a main context of
+    23040 tokens (32 layers, 32 q / 8 kv heads, D 128); fork 4 auxiliary
+    branches; 64 steps in which main and branches append one row and decode
+    (about the paper's branch tokens per turn); harvest the branches' token
+    streams (synthetic ids with thought tags) on the device; merge the
+    harvested rows into main; release the branches.  Three turns (the context
+    grows by each merge); prints the phases of the last two."""
+    import numpy as np
+    import torch
+    import paper_2608_13667_gb300 as st
+    from workloads import Workload, kv_rows, queries
+    dev = torch.device("cuda", 0)
+    st.build()
+    w = Workload(name="agent_turn", n_layers=32, n_q_heads=32, n_kv_heads=8, head_dim=128, n_blocks=2048, seed=6)
+    L, Hkv, D, n_aux, steps, ctx = w.n_layers, w.n_kv_heads, w.head_dim, 4, 64, 23040
+    pool = st.Pool(n_layers=L, n_q_heads=w.n_q_heads, n_kv_heads=Hkv, head_dim=D, n_blocks=w.n_blocks,
+                   seed=w.seed, device=dev, max_seqs=16, max_decode_branches=8, max_splits=32, max_pages=2048)
+    main = pool.seq_create()
+    for c0 in range(0, ctx, PREFIX_CHUNK):
+        n = min(PREFIX_CHUNK, ctx - c0)
+        k, v = kv_rows(w, ("ctx", c0), n, device=dev)
+        pool.append_kv([main], k.view(L, 1, n, Hkv, D), v.view(L, 1, n, Hkv, D))
+    nb = n_aux + 1
+    sk, sv = kv_rows(w, ("step",), nb, device=dev)
+    sk, sv = sk.view(L, nb, 1, Hkv, D), sv.view(L, nb, 1, Hkv, D)
+    sq = queries(w, ("q",), nb, device=dev)
+    o = torch.empty((L, nb, w.n_q_heads, D), dtype=torch.float32, device=dev)
+    lse = torch.empty((L, nb, w.n_q_heads), dtype=torch.float32, device=dev)
+    t_max = n_aux * steps
+    mk, mv = kv_rows(w, ("merge",), t_max, device=dev)
+    mq = queries(w, ("mq",), t_max, device=dev)
+    rng = np.random.default_rng(6)   # the branches' generated ids: thought tags 7 / 8 among other ids
+    s = rng.integers(100, 5000, size=(n_aux, steps)).astype(np.int32)
+    r = rng.random((n_aux, steps))
+    s[r < 0.06] = 7
+    s[(r >= 0.06) & (r < 0.14)] = 8
+    ds = torch.from_numpy(s).to(dev)
+    dl = torch.full((n_aux,), steps, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    turns = []
+    for turn in range(3):
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        br = [main] + pool.fork(main, n_aux)
+        t1 = time.perf_counter()
+        e0, e1 = ev(), ev()
+        e0.record(stream)
+        for _ in range(steps):
+            pool.append_kv(br, sk, sv)
+            pool.decode_attn(br, sq, o, lse)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)   # the observation arrives: the branches stop here
+        th0 = time.perf_counter()
+        ids, src, atoms = st.st_harvest(ds, dl, 7, 8, 5)   # reads the count back: the host sizes the merge
+        T = int(ids.numel())
+        th1 = time.perf_counter()
+        qT, kT, vT = (x[:, :T].contiguous() for x in (mq, mk, mv))   # the thought rows' Q/K/V
+        oT = torch.empty((L, T, w.n_q_heads, D), dtype=torch.float32, device=dev)
+        lT = torch.empty((L, T, w.n_q_heads), dtype=torch.float32, device=dev)
+        e2, e3 = ev(), ev()
+        e2.record(stream)
+        if T:
+            pool.merge(main, qT, kT, vT, oT, lT)
+        e3.record(stream)
+        torch.cuda.synchronize(dev)
+        t2 = time.perf_counter()
+        for b in br[1:]:
+            pool.release(b)
+        t3 = time.perf_counter()
+        turns.append({"context_tokens": pool.block_table(main)[1], "fork_us": (t1 - t0) * 1e6,
+                      "decode_ms": e0.elapsed_time(e1), "decode_us_per_step": e0.elapsed_time(e1) / steps * 1e3,
+                      "harvest_us_with_readback": (th1 - th0) * 1e6, "harvested_rows": T,
+                      "merge_ms": e2.elapsed_time(e3), "release_us": (t3 - t2) * 1e6, "turn_ms": (t3 - t0) * 1e3})
+    pool.sync()
+    pool.close()
+    print(json.dumps({"workload": "one agent turn: 23040-token main, 32 layers, 4 aux branches, 64 steps",
+                      "turns": turns[1:]}))
+
+
 def run_harvest():
     """The thought harvest (st_harvest) on token ids: 4 branches x 512 generated
     tokens (one turn's aux branches at the cycle's 512 steps) and 32 x 2048.
@@ -753,6 +834,8 @@ def main():
                     help="run the small decode + merge case used for ncu captures and exit")
     ap.add_argument("--profile-wide", action="store_true",
                     help="run the small 9-branch decode case (wide tile) used for ncu captures and exit")
+    ap.add_argument("--turn", action="store_true",
+                    help="time one agent turn (fork, 64 decode steps, harvest, merge, release) and exit")
     ap.add_argument("--harvest", action="store_true",
                     help="time the thought harvest (st_harvest) and exit")
     ap.add_argument("--prefill-batch", action="store_true",
@@ -773,6 +856,9 @@ def main():
         return
     if args.harvest:
         run_harvest()
+        return
+    if args.turn:
+        run_turn()
         return
     if args.profile_wide:
         run_profile_wide()
