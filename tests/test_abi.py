@@ -50,3 +50,23 @@ def test_status_strings(stlib):
     L = stlib.lib()
     for s in range(6):
         assert L.st_status_str(s)
+
+
+def test_header_is_plain_c(tmp_path):
+    """include/st.h is a C header (no C++ in the signatures): a C99 program
+    that takes the address of every declared entry point compiles warning-free,
+    and so does the same file as C++."""
+    import shutil
+    import pytest
+    if not shutil.which("gcc"):
+        pytest.skip("no C compiler")
+    names = _declared()
+    src = tmp_path / "use_st.c"
+    src.write_text('#include "st.h"\n#include <stdio.h>\ntypedef void (*fn_t)(void);\nint main(void) {\n'
+                   "  fn_t fns[] = {" + ", ".join(f"(fn_t)&{n}" for n in names) + "};\n"
+                   '  printf("%d\\n", (int)(sizeof fns / sizeof fns[0]));\n  return 0;\n}\n')
+    inc = os.path.join(ROOT, "include")
+    for cmd in (["gcc", "-std=c99", "-Wall", "-Wextra", "-Wpedantic", "-Werror", "-fsyntax-only"],
+                ["g++", "-std=c++17", "-Wall", "-Werror", "-fsyntax-only", "-x", "c++"]):
+        r = subprocess.run(cmd + ["-I", inc, str(src)], capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
