@@ -17,7 +17,14 @@
  *
  * Conventions for every call:
  *  - Return value: ST_OK or an error code; a failing call changes no state.
- *    st_last_error() gives a one-line reason for the last failure.
+ *    st_last_error() gives a one-line reason for the last failure.  The one
+ *    exception is a CUDA call that fails after an append has changed the
+ *    host tables (st_append_kv, st_merge, st_prefill_batch; or the table
+ *    upload at the start of st_decode_attn): that call returns ST_ERR_CUDA
+ *    and the pool is then unusable -- every later call on it returns
+ *    ST_ERR_STATE except st_pool_destroy, st_last_error and the
+ *    introspection calls (st_block_table, st_refcounts, st_free_list,
+ *    st_decode_plan, st_profile_*), which report the host's view.
  *  - Device pointers are plain CUDA device addresses on the pool's device;
  *    the caller owns them (KV storage, workspace, inputs, outputs).
  *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls that
@@ -64,6 +71,10 @@ typedef int64_t st_seq;
  * faulting, and the next st_sync reports ST_ERR_TIMEOUT.  Outputs of such a
  * call are undefined.  Never set in normal use. */
 #define ST_FLAG_HOLD_LOADS 1
+/* Test hook for the CUDA-failure path: with this flag every kernel launch
+ * the pool would make is skipped and reported as failed (ST_ERR_CUDA), as a
+ * failing launch would be.  Never set in normal use. */
+#define ST_FLAG_FAIL_LAUNCH 2
 typedef struct st_pool st_pool;
 
 /* Pool geometry and capacities.
@@ -258,6 +269,10 @@ typedef struct {
   double flops;        /* algorithmic floating-point operations */
   int64_t kernels;     /* device kernels launched (a decode call with both tile
                           shapes launches two per call) */
+  double overhead_bytes; /* bytes moved beyond the algorithmic ones: split-KV
+                            partials (written by the decode, read by the
+                            combine), second reads of a split fork family's
+                            shared pages, copy-on-write rows */
 } st_kernel_stat;
 ST_API st_status st_profile_enable(st_pool* pool, int enable);
 ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, int* n);

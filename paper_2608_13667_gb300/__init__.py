@@ -17,6 +17,7 @@ from ._build import LIB, build  # noqa: F401
 
 ST_OK, ST_ERR_INVALID, ST_ERR_OOM, ST_ERR_STATE, ST_ERR_CUDA, ST_ERR_TIMEOUT = range(6)
 ST_FLAG_HOLD_LOADS = 1
+ST_FLAG_FAIL_LAUNCH = 2
 PAGE = 16
 
 
@@ -51,6 +52,7 @@ class StKernelStat(ctypes.Structure):
         ("bytes", ctypes.c_double),
         ("flops", ctypes.c_double),
         ("kernels", ctypes.c_int64),
+        ("overhead_bytes", ctypes.c_double),
     ]
 
 
@@ -361,7 +363,8 @@ class Pool:
         n = ctypes.c_int()
         self._check(lib().st_profile_read(self._h, buf, 16, ctypes.byref(n)), "st_profile_read")
         return {buf[i].name.decode(): dict(launches=buf[i].launches, total_ms=buf[i].total_ms,
-                                           bytes=buf[i].bytes, flops=buf[i].flops, kernels=buf[i].kernels)
+                                           bytes=buf[i].bytes, flops=buf[i].flops, kernels=buf[i].kernels,
+                                           overhead_bytes=buf[i].overhead_bytes)
                 for i in range(n.value)}
 
 

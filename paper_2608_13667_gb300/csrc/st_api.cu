@@ -15,6 +15,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <initializer_list>
 #include <map>
 #include <tuple>
 #include <new>
@@ -91,6 +92,7 @@ struct KStat {
   int64_t launches = 0;  // calls of this kind
   int64_t kernels = 0;   // device kernels they launched
   double ms = 0, bytes = 0, flops = 0;
+  double overhead_bytes = 0;  // moved beyond the algorithmic bytes (split-KV partials, sibling re-reads)
 };
 
 struct PendingTiming {
@@ -138,6 +140,10 @@ struct st_pool {
   cudaEvent_t stage_ev[kStageSlots] = {};
   bool stage_used[kStageSlots] = {};
   int stage_next = 0;
+  uint32_t stage_held = 0;  // slots taken by a call that has not retired them yet
+  // Set when a CUDA call failed after the host tables had changed: the device
+  // copy may then disagree with them, so every later call is refused.
+  bool broken = false;
   // accounting
   bool timing = false;
   KStat stats[kNumKernels];
@@ -207,18 +213,34 @@ cudaEvent_t take_event(st_pool* P) {
   return e;
 }
 
+// Marks the pool unusable after a failure that left host and device state
+// apart (a CUDA error once the host tables had changed).
+st_status poison(st_pool* P, st_status s) {
+  P->broken = true;
+  P->err = "pool unusable after: " + P->err;
+  return s;
+}
+
+// Every call that changes or reads pool state starts here.
+st_status refuse_if_broken(st_pool* P) {
+  if (!P->broken) return ST_OK;
+  P->err = "the pool is unusable after an earlier CUDA failure; destroy it";
+  return ST_ERR_STATE;
+}
+
 // Launch wrapper: counts the launch (and the n_kernels device kernels it
-// makes), adds its algorithmic bytes/flops, and brackets it with events when
-// timing is on.
+// makes), adds its algorithmic bytes/flops and the bytes it moves beyond
+// them, and brackets it with events when timing is on.  With
+// ST_FLAG_FAIL_LAUNCH the launch is not made and reported as failed.
 template <class F>
 st_status run_kernel(st_pool* P, int kid, double bytes, double flops, cudaStream_t s, F&& launch,
-                     int n_kernels = 1) {
+                     int n_kernels = 1, double overhead_bytes = 0) {
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (P->timing) {
     e0 = take_event(P);
     cudaEventRecord(e0, s);
   }
-  const cudaError_t e = launch();
+  const cudaError_t e = (P->cfg.flags & ST_FLAG_FAIL_LAUNCH) ? cudaErrorLaunchFailure : launch();
   if (e != cudaSuccess)
     return fail(P, ST_ERR_CUDA, "%s launch failed: %s", kKernelNames[kid], cudaGetErrorString(e));
   if (P->timing) {
@@ -231,14 +253,19 @@ st_status run_kernel(st_pool* P, int kid, double bytes, double flops, cudaStream
   k.kernels += n_kernels;
   k.bytes += bytes;
   k.flops += flops;
+  k.overhead_bytes += overhead_bytes;
   return ST_OK;
 }
 
-// Takes the next staging slot, waiting for the work that last used it.
+// Takes the next staging slot that no unfinished call holds, waiting for the
+// work that last used it.  The slot stays held until retire_plan or
+// drop_plan.
 st_status acquire_plan(st_pool* P, Plan* plan, int* slot_out) {
-  const int i = P->stage_next;
+  int i = P->stage_next;
+  while (P->stage_held & (1u << i)) i = (i + 1) % kStageSlots;  // at most two are ever held
   P->stage_next = (i + 1) % kStageSlots;
   if (P->stage_used[i]) CUDA_TRY(P, cudaEventSynchronize(P->stage_ev[i]));
+  P->stage_held |= 1u << i;
   plan->h = P->h_stage + (size_t)i * kStageSlotBytes;
   plan->d = P->ws + P->lay.staging + (size_t)i * kStageSlotBytes;
   plan->cap = kStageSlotBytes;
@@ -253,9 +280,22 @@ st_status submit_plan(st_pool* P, const Plan& plan, cudaStream_t s) {
 }
 
 st_status retire_plan(st_pool* P, int slot, cudaStream_t s) {
+  P->stage_held &= ~(1u << slot);
   CUDA_TRY(P, cudaEventRecord(P->stage_ev[slot], s));
   P->stage_used[slot] = true;
   return ST_OK;
+}
+
+// Gives back a slot that was taken but never written to the device.
+void drop_plan(st_pool* P, int slot) {
+  if (slot >= 0) P->stage_held &= ~(1u << slot);
+}
+
+// Bytes a plan of these arrays takes in a staging slot (16-byte aligned parts).
+size_t plan_bytes(std::initializer_list<size_t> parts) {
+  size_t off = 0;
+  for (size_t b : parts) off = align_up(off, 16) + b;
+  return off;
 }
 
 // Refresh the device copy of every block-table range the host changed.
@@ -313,14 +353,17 @@ st_status flush_tables(st_pool* P, cudaStream_t s) {
 
 bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
-// Validates and performs an append (shared by st_append_kv and st_merge).
-// Appends counts[i] rows to slots[i], in order (the same page allocation as
-// appending to each sequence in turn); k, v: [L][sum of counts][Hkv][D].
-// All or nothing: capacity is checked before any table changes.
+// Validates and performs an append (shared by st_append_kv, st_merge and
+// st_prefill_batch).  Appends counts[i] rows to slots[i], in order (the same
+// page allocation as appending to each sequence in turn); k, v: [L][sum of
+// counts][Hkv][D].  All or nothing: capacity, the plan's size and its staging
+// slot are settled before any table changes; a CUDA failure after that
+// leaves the pool unusable (every later call returns ST_ERR_STATE).
 st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, int n_br, const void* k,
                          const void* v, cudaStream_t s) {
   BlockPool& bp = *P->pool;
   int64_t need = 0, n_rows = 0;
+  int cow_bound = 0;  // branches whose append may start with a copy-on-write
   bool uniform = true;
   for (int i = 0; i < n_br; ++i) {
     if (!bp.fits(slots[i], counts[i]))
@@ -328,11 +371,28 @@ st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, in
     need += bp.pages_needed(slots[i], counts[i]);
     n_rows += counts[i];
     uniform = uniform && counts[i] == counts[0];
+    const SeqSlot& ss = bp.slot(slots[i]);
+    if (counts[i] > 0 && ss.len % kPageTokens != 0 && bp.refcounts()[ss.table.back()] > 1) ++cow_bound;
   }
   if (need > bp.free_count())
     return fail(P, ST_ERR_OOM, "pool has %lld free pages, call needs %lld",
                 (long long)bp.free_count(), (long long)need);
   if (n_rows > INT32_MAX) return fail(P, ST_ERR_INVALID, "too many rows in one call");
+  // Small plans travel in the kernel parameters, larger ones through a
+  // staging slot.  Copy-on-writes can only be fewer than cow_bound (an
+  // earlier branch's copy may leave a later one the last holder).
+  const bool may_stage = n_rows > 0 && !(n_br <= kInlineAppendBranches && cow_bound <= kInlineCows);
+  if (may_stage && plan_bytes({n_br * sizeof(AppendBranch), std::max(cow_bound, 1) * sizeof(CowCopy)}) >
+                       kStageSlotBytes)
+    return fail(P, ST_ERR_INVALID, "append of %d sequences does not fit one plan slot", n_br);
+  Plan plan;
+  int ps = -1;
+  if (may_stage && !P->meta_only) {
+    st_status st = acquire_plan(P, &plan, &ps);
+    if (st != ST_OK) return st;
+  }
+
+  // ---- from here on the host tables change ----------------------------------
   std::vector<AppendBranch> brs(n_br);
   int32_t row0 = 0;
   for (int i = 0; i < n_br; ++i) {
@@ -348,29 +408,25 @@ st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, in
   if (P->meta_only || n_rows == 0) return ST_OK;
 
   st_status st = flush_tables(P, s);
-  if (st != ST_OK) return st;
-  // small plans travel in the kernel parameters; larger ones through staging
+  if (st != ST_OK) return poison(P, st);
   const bool inline_plan = n_br <= kInlineAppendBranches && cows.size() <= (size_t)kInlineCows;
   InlineAppendPlan inl;
   const AppendBranch* d_br = nullptr;
   const CowCopy* d_cow = nullptr;
-  Plan plan;
-  int ps = -1;
   if (inline_plan) {
+    drop_plan(P, ps);
+    ps = -1;
     for (int i = 0; i < n_br; ++i) inl.branches[i] = brs[i];
     for (size_t i = 0; i < cows.size(); ++i)
       inl.cows[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
   } else {
-    st = acquire_plan(P, &plan, &ps);
-    if (st != ST_OK) return st;
     AppendBranch* br = plan.alloc<AppendBranch>(n_br, &d_br);
     CowCopy* cw = plan.alloc<CowCopy>(std::max<size_t>(cows.size(), 1), &d_cow);
-    if (!br || !cw) return fail(P, ST_ERR_INVALID, "append plan does not fit the staging slot");
     for (int i = 0; i < n_br; ++i) br[i] = brs[i];
     for (size_t i = 0; i < cows.size(); ++i)
       cw[i] = CowCopy{cows[i].src_block, cows[i].dst_block, cows[i].rows, 0};
     st = submit_plan(P, plan, s);
-    if (st != ST_OK) return st;
+    if (st != ST_OK) return poison(P, st);
   }
   const st_config& c = P->cfg;
   AppendParams ap{};
@@ -391,14 +447,20 @@ st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, in
   ap.max_pages = c.max_pages;
   ap.n_rows = (int32_t)n_rows;
   ap.ragged = uniform ? 0 : 1;
+  // algorithmic: the new rows read and written once; the copy-on-write rows
+  // are the bookkeeping's own traffic
   const double row_bytes = (double)c.n_layers * c.n_kv_heads * c.head_dim * 2 * 2;
   double cow_rows = 0;
   for (auto& e : cows) cow_rows += e.rows;
-  const double bytes = row_bytes * ((double)n_rows * 2 + cow_rows * 2);
-  st = run_kernel(P, kKAppend, bytes, 0, s,
-                  [&] { return launch_append(ap, inline_plan ? &inl : nullptr, c.head_dim, s); });
-  if (st != ST_OK) return st;
-  return inline_plan ? ST_OK : retire_plan(P, ps, s);
+  st = run_kernel(P, kKAppend, row_bytes * (double)n_rows * 2, 0, s,
+                  [&] { return launch_append(ap, inline_plan ? &inl : nullptr, c.head_dim, s); }, 1,
+                  row_bytes * cow_rows * 2);
+  if (st != ST_OK) return poison(P, st);
+  if (!inline_plan) {
+    st = retire_plan(P, ps, s);
+    if (st != ST_OK) return poison(P, st);
+  }
+  return ST_OK;
 }
 
 st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const void* k, const void* v,
@@ -559,6 +621,7 @@ ST_API st_status st_pool_destroy(st_pool* P) {
 
 ST_API st_status st_seq_create(st_pool* P, st_seq* out) {
   if (!P || !out) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   const int s = P->pool->create_seq();
   if (s < 0) return fail(P, ST_ERR_OOM, "no free sequence slot (max_seqs = %d)", P->cfg.max_seqs);
   *out = make_handle(P, s);
@@ -577,6 +640,7 @@ struct NvtxRange {
 ST_API st_status st_fork(st_pool* P, st_seq seq, int n_aux, st_seq* out_aux) {
   NvtxRange range_("st_fork");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
   return st_fork_at(P, seq, P->pool->slot(slot).len, n_aux, out_aux);
@@ -585,6 +649,7 @@ ST_API st_status st_fork(st_pool* P, st_seq seq, int n_aux, st_seq* out_aux) {
 ST_API st_status st_fork_at(st_pool* P, st_seq seq, int64_t length, int n_aux, st_seq* out_aux) {
   NvtxRange range_("st_fork_at");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
   if (n_aux < 0 || (n_aux > 0 && !out_aux)) return fail(P, ST_ERR_INVALID, "bad n_aux/out_aux");
@@ -602,6 +667,7 @@ ST_API st_status st_fork_at(st_pool* P, st_seq seq, int64_t length, int n_aux, s
 ST_API st_status st_release(st_pool* P, st_seq seq) {
   NvtxRange range_("st_release");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   int slot;
   if (!decode_handle(P, seq, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
   P->pool->release(slot);
@@ -612,6 +678,7 @@ ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok,
                               const void* v, void* stream) {
   NvtxRange range_("st_append_kv");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   if (n_br < 0 || n_tok < 0 || (n_br > 0 && !br)) return fail(P, ST_ERR_INVALID, "bad n_br/n_tok");
   std::vector<int> slots(n_br);
   for (int i = 0; i < n_br; ++i) {
@@ -643,8 +710,12 @@ struct DecodePlan {
   std::vector<AttnItem> items;
   std::vector<int32_t> members;   // the call's branch index of each item's members
   std::vector<int32_t> n_splits;  // partials per branch
-  double bytes = 0, flops = 0;    // algorithmic, whole launch (KV pages, Q, partials)
-  double part_bytes = 0;          // the partials alone (written here, read by the combine)
+  // algorithmic, whole launch: every KV page once per fork family and layer
+  // (shared pages once for the family, own pages once for their branch) and
+  // the queries
+  double bytes = 0, flops = 0;
+  double reread_bytes = 0;        // second and later reads of a split family's pages
+  double part_bytes = 0;          // the split-KV partials (written here, read by the combine)
 };
 
 void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
@@ -654,7 +725,7 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   const int n_br = (int)slots.size();
   // ---- group by fork family, find the shared full pages --------------------
   std::vector<int32_t> shared(n_br, 0);   // pages of branch i read through its group
-  struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split, wide; };
+  struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split, wide, reread; };
   std::vector<Group> groups;
   {
     std::map<int32_t, std::vector<int>> fam;
@@ -699,6 +770,7 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
         g.family = f;
         g.split = n_sub > 1;
         g.wide = wide;
+        g.reread = sg > 0;  // the family's pages were counted with its first subgroup
         for (int i : g.members) shared[i] = pages;
         groups.push_back(std::move(g));
       }
@@ -759,7 +831,7 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   std::vector<int32_t> item_family;  // fork family of a subgroup's item, for scheduling siblings together
   std::vector<int32_t> members;
   std::vector<int32_t> n_splits(n_br, 0);
-  double bytes = 0, flops = 0;
+  double bytes = 0, flops = 0, reread = 0;
   const double page_bytes = (double)kPageTokens * c.head_dim * 2 * 2;  // K+V, one head
   for (auto& g : groups) {
     const int32_t k = (int32_t)std::min<int64_t>(max_prefix_chunks, (g.pages + chunk - 1) / chunk);
@@ -771,7 +843,7 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
       items.push_back(AttnItem{slots[g.members[0]], b, n, n * kPageTokens, mbase, (int32_t)g.members.size(),
                                cidx, (g.split ? kItemReread : 0) | (g.wide ? kItemWide : 0)});
       item_family.push_back(g.family);
-      bytes += n * page_bytes;
+      (g.reread ? reread : bytes) += n * page_bytes;
       flops += 4.0 * g.members.size() * G * n * kPageTokens * c.head_dim;
     }
     for (int i : g.members) n_splits[i] = k;
@@ -812,19 +884,19 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
     items.swap(sorted);
   }
   bytes *= (double)c.n_kv_heads * c.n_layers;
+  reread *= (double)c.n_kv_heads * c.n_layers;
   flops *= (double)c.n_kv_heads * c.n_layers;
   const double q_bytes = (double)c.n_layers * n_br * c.n_q_heads * c.head_dim * 2;
   double part_rows = 0;
   for (auto& it : items) part_rows += (double)it.n_members * G;
   part_rows *= (double)c.n_kv_heads * c.n_layers;
-  const double part_bytes = part_rows * (c.head_dim + 1) * 4;
-  bytes += q_bytes + part_bytes;
   out->items = std::move(items);
   out->members = std::move(members);
   out->n_splits = std::move(n_splits);
-  out->bytes = bytes;
+  out->bytes = bytes + q_bytes;
   out->flops = flops;
-  out->part_bytes = part_bytes;
+  out->reread_bytes = reread;
+  out->part_bytes = part_rows * (c.head_dim + 1) * 4;
 }
 
 // The call's branches as pool slots: live, non-empty, each listed once.
@@ -848,6 +920,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
                                 float* lse, void* stream) {
   NvtxRange range_("st_decode_attn");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
   if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
     return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
@@ -861,16 +934,20 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
 
   DecodePlan dp;
   plan_decode(P, slots, &dp);
-  st_status st = flush_tables(P, s);
-  if (st != ST_OK) return st;
   const std::vector<AttnItem>& items = dp.items;
   const std::vector<int32_t>& members = dp.members;
   const std::vector<int32_t>& n_splits = dp.n_splits;
   const double bytes = dp.bytes, flops = dp.flops, part_bytes = dp.part_bytes;
-
   // small plans travel in the kernel parameters; larger ones through staging
   const bool inline_plan = items.size() <= (size_t)kInlineItems && members.size() <= (size_t)kInlineMembers &&
                            n_br <= kInlineBranches;
+  if (!inline_plan && plan_bytes({items.size() * sizeof(AttnItem), members.size() * sizeof(int32_t),
+                                  n_br * sizeof(int32_t)}) > kStageSlotBytes)
+    return fail(P, ST_ERR_INVALID, "decode plan of %d items does not fit one plan slot", (int)items.size());
+  // device tables that missed an upload would disagree with the host's
+  st_status st = flush_tables(P, s);
+  if (st != ST_OK) return poison(P, st);
+
   InlineDecodePlan inl;
   const AttnItem* d_items = nullptr;
   const int32_t* d_members = nullptr;
@@ -887,12 +964,14 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     AttnItem* hi = plan.alloc<AttnItem>(items.size(), &d_items);
     int32_t* hm = plan.alloc<int32_t>(members.size(), &d_members);
     int32_t* hn = plan.alloc<int32_t>(n_br, &d_nsplit);
-    if (!hi || !hm || !hn) return fail(P, ST_ERR_INVALID, "decode plan does not fit the staging slot");
     std::memcpy(hi, items.data(), items.size() * sizeof(AttnItem));
     std::memcpy(hm, members.data(), members.size() * sizeof(int32_t));
     std::memcpy(hn, n_splits.data(), n_br * sizeof(int32_t));
     st = submit_plan(P, plan, s);
-    if (st != ST_OK) return st;
+    if (st != ST_OK) {
+      drop_plan(P, ps);
+      return st;
+    }
   }
 
   AttnParams ap{};
@@ -926,8 +1005,11 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     AttnParams aw = ap;
     aw.item_base = n_narrow;
     return launch_decode_tc(P->kmap, P->vmap, aw, ip, n_items - n_narrow, c.head_dim, true, s);
-  }, (n_narrow > 0 ? 1 : 0) + (n_items > n_narrow ? 1 : 0));
-  if (st != ST_OK) return st;
+  }, (n_narrow > 0 ? 1 : 0) + (n_items > n_narrow ? 1 : 0), dp.reread_bytes + part_bytes);
+  if (st != ST_OK) {
+    if (ps >= 0) retire_plan(P, ps, s);  // its copy may still be in flight
+    return st;
+  }
 
   CombineParams cp{};
   cp.part_o = P->d_part_o;
@@ -939,10 +1021,14 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   cp.Hq = c.n_q_heads;
   cp.L = c.n_layers;
   cp.max_splits = c.max_splits;
-  const double cbytes = part_bytes + (double)c.n_layers * n_br * c.n_q_heads * (c.head_dim + 1) * 4;
+  // algorithmic: O and LSE written once; the partials it reads are the split's own traffic
+  const double cbytes = (double)c.n_layers * n_br * c.n_q_heads * (c.head_dim + 1) * 4;
   st = run_kernel(P, kKCombine, cbytes, 0, s,
-                  [&] { return launch_combine(cp, inline_plan ? &inl : nullptr, c.head_dim, s); });
-  if (st != ST_OK) return st;
+                  [&] { return launch_combine(cp, inline_plan ? &inl : nullptr, c.head_dim, s); }, 1, part_bytes);
+  if (st != ST_OK) {
+    if (ps >= 0) retire_plan(P, ps, s);  // its copy may still be in flight
+    return st;
+  }
   return inline_plan ? ST_OK : retire_plan(P, ps, s);
 }
 
@@ -983,6 +1069,7 @@ ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, con
                           const void* v, float* o, float* lse, void* stream) {
   NvtxRange range_("st_merge");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   int slot;
   if (!decode_handle(P, main, &slot)) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
   if (n_tok < 0) return fail(P, ST_ERR_INVALID, "n_tok < 0");
@@ -1025,8 +1112,9 @@ ST_API st_status st_merge(st_pool* P, st_seq main, int n_tok, const void* q, con
   const double io_bytes = (double)c.n_layers * n_tok * c.n_q_heads * (c.head_dim * 2 + c.head_dim * 4 + 4);
   const double keys = (double)n_tok * L0 + (double)n_tok * (n_tok + 1) / 2;
   const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
-  return run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
-                    [&] { return launch_merge_tc(P->kmap, P->vmap, ap, 0, c.head_dim, s); });
+  st = run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
+                  [&] { return launch_merge_tc(P->kmap, P->vmap, ap, 0, c.head_dim, s); });
+  return st == ST_OK ? ST_OK : poison(P, st);  // the rows are in, their prefill is not
 }
 
 ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, const int32_t* n_tok,
@@ -1034,6 +1122,7 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
                                   void* stream) {
   NvtxRange range_("st_prefill_batch");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   if (n_seq < 0 || (n_seq > 0 && (!seqs || !n_tok))) return fail(P, ST_ERR_INVALID, "bad n_seq/seqs/n_tok");
   std::vector<int> slots;
   std::vector<int32_t> counts;
@@ -1051,6 +1140,13 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
     }
   }
   if (R > INT32_MAX) return fail(P, ST_ERR_INVALID, "too many rows in one call");
+  const st_config& c = P->cfg;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  // work items: each sequence's stacked (row, head) rows in tiles of 256
+  int64_t n_items64 = 0;
+  for (size_t i = 0; i < slots.size(); ++i) n_items64 += ((int64_t)counts[i] * G + 255) / 256;
+  if (plan_bytes({(size_t)n_items64 * sizeof(MergeItem)}) > kStageSlotBytes)
+    return fail(P, ST_ERR_INVALID, "prefill of %lld row tiles does not fit one plan slot", (long long)n_items64);
   if (P->meta_only) {
     if (q || k || v || o || lse) return fail(P, ST_ERR_INVALID, "metadata-only pool takes no data");
     return do_append_rows(P, slots.data(), counts.data(), (int)slots.size(), nullptr, nullptr, nullptr);
@@ -1059,16 +1155,11 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
   if (!q || !k || !v || !o || !lse || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) ||
       !aligned(o, 16) || !aligned(lse, 4))
     return fail(P, ST_ERR_INVALID, "q/k/v/o/lse must be aligned device pointers");
-  const st_config& c = P->cfg;
-  const int G = c.n_q_heads / c.n_kv_heads;
   std::vector<int32_t> L0(slots.size());
   for (size_t i = 0; i < slots.size(); ++i) L0[i] = (int32_t)P->pool->slot(slots[i]).len;
   DeviceGuard guard(P->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  st_status st = do_append_rows(P, slots.data(), counts.data(), (int)slots.size(), k, v, s);
-  if (st != ST_OK) return st;
 
-  // work items: each sequence's stacked (row, head) rows in tiles of 256
   std::vector<MergeItem> items;
   double kv_bytes = 0, io_bytes = 0, keys = 0;
   int32_t q_row0 = 0;
@@ -1090,14 +1181,18 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
   const double flops = 4.0 * c.head_dim * keys * c.n_q_heads * c.n_layers;
   Plan plan;
   int ps = -1;
-  st = acquire_plan(P, &plan, &ps);
+  st_status st = acquire_plan(P, &plan, &ps);
   if (st != ST_OK) return st;
+  st = do_append_rows(P, slots.data(), counts.data(), (int)slots.size(), k, v, s);
+  if (st != ST_OK) {
+    drop_plan(P, ps);  // nothing was written to it
+    return st;
+  }
   const MergeItem* d_items = nullptr;
   MergeItem* hi = plan.alloc<MergeItem>(items.size(), &d_items);
-  if (!hi) return fail(P, ST_ERR_INVALID, "prefill plan does not fit the staging slot");
   std::memcpy(hi, items.data(), items.size() * sizeof(MergeItem));
   st = submit_plan(P, plan, s);
-  if (st != ST_OK) return st;
+  if (st != ST_OK) return poison(P, st);
   AttnParams ap{};
   ap.q = static_cast<const __nv_bfloat16*>(q);
   ap.out_o = o;
@@ -1118,8 +1213,9 @@ ST_API st_status st_prefill_batch(st_pool* P, const st_seq* seqs, int n_seq, con
   const int n_items = (int)items.size();
   st = run_kernel(P, kKMerge, kv_bytes + io_bytes, flops, s,
                   [&] { return launch_merge_tc(P->kmap, P->vmap, ap, n_items, c.head_dim, s); });
-  if (st != ST_OK) return st;
-  return retire_plan(P, ps, s);
+  const st_status rs = retire_plan(P, ps, s);
+  if (st != ST_OK) return poison(P, st);
+  return rs == ST_OK ? ST_OK : poison(P, rs);
 }
 
 ST_API st_status st_block_table(st_pool* P, st_seq seq, int32_t* out, int cap, int* n_pages,
@@ -1157,6 +1253,7 @@ ST_API st_status st_free_list(st_pool* P, int32_t* out, int64_t cap, int64_t* n)
 ST_API st_status st_sync(st_pool* P, void* stream) {
   NvtxRange range_("st_sync");
   if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
   if (P->meta_only) return ST_OK;
   DeviceGuard guard(P->device);
   CUDA_TRY(P, cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
@@ -1200,6 +1297,7 @@ ST_API st_status st_profile_read(st_pool* P, st_kernel_stat* out, int cap, int* 
       out[k].bytes = P->stats[i].bytes;
       out[k].flops = P->stats[i].flops;
       out[k].kernels = P->stats[i].kernels;
+      out[k].overhead_bytes = P->stats[i].overhead_bytes;
       ++k;
     }
     P->stats[i] = KStat{};

@@ -91,3 +91,34 @@ def test_pool_exhaustion_mid_decode_loop(stlib):
     o_ref, l_ref = run.oracle_decode(br, q, 0)
     compare(o[0], lse[0], o_ref, l_ref, "after exhaustion")
     run.check_tables()
+
+
+def test_failed_launch_after_append_makes_the_pool_unusable(stlib):
+    # ST_FLAG_FAIL_LAUNCH reports every launch as failed without making it (a
+    # fake of a failing CUDA launch): the append has already changed the host
+    # tables when its launch fails, so the pool refuses every later call.
+    pool = stpkg.Pool(n_layers=1, n_q_heads=8, n_kv_heads=2, head_dim=64, n_blocks=32, seed=3,
+                      max_seqs=4, device="cuda", flags=stpkg.ST_FLAG_FAIL_LAUNCH)
+    m = pool.seq_create()
+    kv = torch.zeros((1, 1, 20, 2, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(stpkg.STError) as e:
+        pool.append_kv([m], kv, kv)
+    assert e.value.status == stpkg.ST_ERR_CUDA
+    for call in (lambda: pool.append_kv([m], kv, kv), lambda: pool.fork(m, 2), pool.seq_create,
+                 lambda: pool.release(m), pool.sync,
+                 lambda: pool.decode_attn([m], torch.zeros((1, 1, 8, 64), dtype=torch.bfloat16, device="cuda"))):
+        with pytest.raises(stpkg.STError) as e:
+            call()
+        assert e.value.status == stpkg.ST_ERR_STATE
+        assert "unusable" in str(e.value)
+    # introspection still reports the host's view: the 20 rows went in
+    assert pool.block_table(m)[1] == 20
+    pool.close()
+    # a pool without the flag on the same device is unaffected
+    run = Run(_w(), max_seqs=4, max_decode_branches=2, max_splits=4)
+    a = run.create()
+    run.append([a], 21, ("ctx",))
+    q, o, lse = run.decode([a], ("q",))
+    run.pool.sync()
+    o_ref, l_ref = run.oracle_decode([a], q, 0)
+    compare(o[0], lse[0], o_ref, l_ref, "after a broken pool")
