@@ -193,3 +193,68 @@ def test_fork_at_mid_page_copies_on_first_append():
     assert len(ev) == 1 and ev[0][0] == pool.seqs[m].table[1] and ev[0][2] == 5
     assert pool.read(c) == [("m", i) for i in range(21)] + [("c", 0)]
     assert pool.read(m) == [("m", i) for i in range(40)]
+
+
+def _fork_family(seed):
+    """main with 37 rows (a partial third page) and three forks of it, plus a
+    fresh sequence: content tracked, labels (sequence, row)."""
+    pool = P.RefPool(n_blocks=64, seed=seed, track_content=True)
+    m = pool.create()
+    pool.append([m], 37, [[("m", i) for i in range(37)]])
+    kids = pool.fork(m, 3)
+    fresh = pool.create()
+    return pool, [m] + kids + [fresh]
+
+
+def test_ragged_prefill_equals_appends_one_by_one():
+    counts = [5, 0, 27, 1, 40]     # unequal; one empty; copies of the shared partial page
+    a, ids = _fork_family(8)
+    b, _ = _fork_family(8)
+    labels = [[(i, t) for t in range(n)] for i, n in zip(ids, counts)]
+    ev_batch = a.prefill_batch(ids, counts, labels)
+    ev_single = []
+    for i, n, lab in zip(ids, counts, labels):
+        ev_single += b.prefill_batch([i], [n], [lab])
+    assert ev_batch == ev_single
+    assert [a.seqs[i].table for i in ids] == [b.seqs[i].table for i in ids]
+    assert [a.seqs[i].length for i in ids] == [37 + 5, 37, 37 + 27, 37 + 1, 40]
+    assert a.ref == b.ref and list(a.free) == list(b.free)
+    # every sequence reads back its own rows after its history, nobody else's
+    hist = {ids[0]: [("m", r) for r in range(37)]}
+    for k in ids[1:4]:
+        hist[k] = [("m", r) for r in range(37)]
+    hist[ids[4]] = []
+    for i, lab in zip(ids, labels):
+        assert a.read(i) == hist[i] + lab
+    _check_invariants(a)
+
+
+def test_ragged_prefill_copies_the_shared_page_only_for_sequences_that_grow():
+    pool, ids = _fork_family(2)
+    shared = pool.seqs[ids[0]].table[2]
+    ev = pool.prefill_batch(ids[:4], [0, 3, 0, 1])
+    # the two growing forks copy rows [0, 5) of the shared third page; the
+    # main thread and the idle fork keep referencing it
+    assert [e[0] for e in ev] == [shared, shared] and all(e[2] == 5 for e in ev)
+    assert pool.ref[shared] == 2
+    assert pool.seqs[ids[0]].table[2] == pool.seqs[ids[2]].table[2] == shared
+
+
+def test_ragged_prefill_capacity_is_checked_for_the_whole_call():
+    # 10 pages; after a = 5 rows (1 page) and b = 17 rows (2 pages) 7 are free.
+    # [12, 20, 96] needs 1 + 1 + 6 = 8 pages: refused, nothing changes.
+    # [12, 20, 80] needs 1 + 1 + 5 = 7 pages: taken, the free list empties.
+    pool = P.RefPool(n_blocks=10, seed=4, track_content=True)
+    a, b, c = pool.create(), pool.create(), pool.create()
+    pool.prefill_batch([a, b, c], [5, 17, 0])
+    assert len(pool.free) == 7
+    snap = (list(pool.ref), list(pool.free), [list(pool.seqs[i].table) for i in (a, b, c)],
+            [pool.seqs[i].length for i in (a, b, c)])
+    with pytest.raises(P.OutOfBlocks):
+        pool.prefill_batch([a, b, c], [12, 20, 96])
+    assert snap == (list(pool.ref), list(pool.free), [list(pool.seqs[i].table) for i in (a, b, c)],
+                    [pool.seqs[i].length for i in (a, b, c)])
+    pool.prefill_batch([a, b, c], [12, 20, 80])
+    assert len(pool.free) == 0
+    assert [len(pool.seqs[i].table) for i in (a, b, c)] == [2, 3, 5]
+    _check_invariants(pool)
