@@ -747,75 +747,157 @@ def run_cycle():
 
 # --------------------------------------------------------------------------- oracle
 
-def oracle_sample_step(w, dev, layer, task=0):
-    """The float64 oracle over one layer of one fork group (all its branches): a
-    bounded sample of the step.  Returns (seconds of oracle work, branch-steps)."""
+def _oracle_worker(w, dev_name, cmd_q, res_q, barrier):
+    """A host-core worker of the oracle baseline.  Per round it receives a
+    list of (layer, KV head) units of fork group 0, draws their inputs (not
+    timed), waits at the barrier with the other workers, then runs the float64
+    oracle (oracle.attention.decode, unchanged) on each unit's branches --
+    every branch's query heads of that KV head over its materialised context,
+    prefix ++ suffix -- and reports its start and end on the monotonic clock."""
     import torch
+    torch.set_num_threads(1)
     from oracle import attention as A
     from workloads import kv_rows, queries
-    ks, vs = [], []
-    for c0 in range(0, w.prefix[task], PREFIX_CHUNK):
-        n = min(PREFIX_CHUNK, w.prefix[task] - c0)
-        k, v = kv_rows(w, ("prefix", task, c0), n, device=dev, layers=[layer])
-        ks.append(k[0].cpu())
-        vs.append(v[0].cpu())
-    pk, pv = torch.cat(ks), torch.cat(vs)
-    q = queries(w, ("q", 0, 0), w.n_aux + 1, device=dev, layers=[layer])[0].cpu()
-    ctx = []
-    for b, s in enumerate(w.suffix[task]):
-        if s:
-            k, v = kv_rows(w, ("suffix", task, b), s, device=dev, layers=[layer])
-            ctx.append((torch.cat([pk, k[0].cpu()]), torch.cat([pv, v[0].cpu()])))
-        else:
-            ctx.append((pk, pv))
-    t0 = time.perf_counter()
-    for b in range(w.n_aux + 1):
-        A.decode(q[b], *ctx[b])
-    dt = time.perf_counter() - t0
-    return dt, (w.n_aux + 1) / w.n_layers
+    dev = torch.device(dev_name)
+    G = w.n_q_heads // w.n_kv_heads
+    while True:
+        units = cmd_q.get()
+        if units is None:
+            return
+        jobs, drawn = [], {}
+        for layer, g in units:
+            if layer not in drawn:
+                ks, vs = [], []
+                for c0 in range(0, w.prefix[0], PREFIX_CHUNK):
+                    n = min(PREFIX_CHUNK, w.prefix[0] - c0)
+                    k, v = kv_rows(w, ("prefix", 0, c0), n, device=dev, layers=[layer])
+                    ks.append(k[0].cpu())
+                    vs.append(v[0].cpu())
+                suf = []
+                for b, n in enumerate(w.suffix[0]):
+                    if n:
+                        k, v = kv_rows(w, ("suffix", 0, b), n, device=dev, layers=[layer])
+                        suf.append((k[0].cpu(), v[0].cpu()))
+                    else:
+                        suf.append(None)
+                q = queries(w, ("q", 0, 0), w.n_aux + 1, device=dev, layers=[layer])[0].cpu()
+                drawn = {layer: (torch.cat(ks), torch.cat(vs), suf, q)}
+            pk, pv, suf, q = drawn[layer]
+            for b in range(w.n_aux + 1):
+                kc, vc = pk[:, g:g + 1], pv[:, g:g + 1]
+                if suf[b] is not None:
+                    kc = torch.cat([kc, suf[b][0][:, g:g + 1]])
+                    vc = torch.cat([vc, suf[b][1][:, g:g + 1]])
+                jobs.append((q[b, g * G:(g + 1) * G].clone(), kc.contiguous(), vc.contiguous()))
+        drawn = {}
+        barrier.wait()
+        t0 = time.monotonic()
+        for qh, kc, vc in jobs:
+            A.decode(qh, kc, vc)
+        t1 = time.monotonic()
+        res_q.put((t0, t1, len(units)))
 
 
-CPU_SAMPLE_S = 10.0  # oracle seconds the cpu_baseline sample aims for (whole layers, at most 30 s)
+class ParallelOracle:
+    """The float64 oracle on the host cores: one spawned worker process per
+    core, each with one BLAS / torch thread, over (layer, KV head) units of
+    one fork group.  A round's time is from the first worker's start to the
+    last worker's end, all workers starting together after drawing their
+    inputs."""
+
+    def __init__(self, w, n_workers=None):
+        import multiprocessing as mp
+        import torch
+        self.w = w
+        self.n = max(1, min(n_workers or os.cpu_count() or 1, w.n_layers * w.n_kv_heads))
+        ctx = mp.get_context("spawn")
+        self.barrier = ctx.Barrier(self.n + 1)
+        self.res = ctx.Queue()
+        self.cmds = [ctx.Queue() for _ in range(self.n)]
+        dev = "cuda" if torch.cuda.is_available() else "cpu"
+        saved = {v: os.environ.get(v) for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS")}
+        os.environ.update({v: "1" for v in saved})
+        try:
+            self.procs = [ctx.Process(target=_oracle_worker, args=(w, dev, q, self.res, self.barrier), daemon=True)
+                          for q in self.cmds]
+            for p in self.procs:
+                p.start()
+        finally:
+            for v, val in saved.items():
+                if val is None:
+                    os.environ.pop(v, None)
+                else:
+                    os.environ[v] = val
+        self.next_unit = 0
+
+    def round(self, units_per_worker):
+        """Runs the next units_per_worker units on every worker; returns
+        (seconds, branch-steps)."""
+        w = self.w
+        all_units = [(l, g) for l in range(w.n_layers) for g in range(w.n_kv_heads)]
+        for q in self.cmds:
+            mine = [all_units[(self.next_unit + i) % len(all_units)] for i in range(units_per_worker)]
+            self.next_unit += units_per_worker
+            q.put(mine)
+        self.barrier.wait()
+        t0, t1, n = [], [], 0
+        for _ in self.procs:
+            a, b, k = self.res.get()
+            t0.append(a)
+            t1.append(b)
+            n += k
+        return max(t1) - min(t0), n * (w.n_aux + 1) / (w.n_layers * w.n_kv_heads)
+
+    def close(self):
+        for q in self.cmds:
+            q.put(None)
+        for p in self.procs:
+            p.join(timeout=30)
 
 
-def cpu_baseline(w, dev):
-    """The oracle on the host cores over a bounded sample of the step: whole
-    layers of one fork group, added until about CPU_SAMPLE_S seconds of oracle
-    work."""
-    dt = units = 0.0
-    layers = 0
-    while layers < w.n_layers and dt < CPU_SAMPLE_S:
-        d, u = oracle_sample_step(w, dev, layer=layers)
-        dt += d
-        units += u
-        layers += 1
-    return {"value": units / dt, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{layers} of {w.n_layers} layers of 1 of {w.n_tasks} fork groups ({w.n_aux + 1} branches, "
-                      f"{w.prefix[0]}-token prefix), float64 numpy; {dt:.1f} s of oracle work"}
+def cpu_baseline(w, n_workers=None):
+    """The oracle on the host cores over a bounded sample of the step: 8
+    layers of one fork group, every KV head, all its branches, spread over
+    one worker per core."""
+    po = ParallelOracle(w, n_workers)
+    try:
+        per = max(1, (min(8, w.n_layers) * w.n_kv_heads) // po.n)
+        dt, units = po.round(per)
+    finally:
+        po.close()
+    n_units = per * po.n
+    layers = min(w.n_layers, -(-n_units // w.n_kv_heads))
+    return {"value": units / dt, "unit": UNIT, "cores": po.n, "kind": "oracle",
+            "sample": f"{n_units} (layer, KV head) units over {layers} of {w.n_layers} layers of 1 of "
+                      f"{w.n_tasks} fork groups ({w.n_aux + 1} branches, {w.prefix[0]}-token prefix), float64 numpy, "
+                      f"{po.n} worker processes with one thread each; {dt:.2f} s wall ({dt * po.n:.1f} core-s)"}
 
 
 def run_reference(args, rank, ws, local):
-    import torch
     w = _workload(args)
     if rank != 0:
         return {}
-    dev = torch.device("cuda", local) if torch.cuda.is_available() else torch.device("cpu")
-    for s in range(args.warmup):
-        oracle_sample_step(w, dev, layer=s % w.n_layers)
-    total_dt = total_units = 0.0
-    for s in range(args.steps):
-        dt, units = oracle_sample_step(w, dev, layer=(args.warmup + s) % w.n_layers)
-        total_dt += dt
-        total_units += units
+    po = ParallelOracle(w, args.oracle_workers)
+    try:
+        for s in range(args.warmup):
+            po.round(1)
+        total_dt = total_units = 0.0
+        for s in range(args.steps):
+            dt, units = po.round(1)
+            total_dt += dt
+            total_units += units
+    finally:
+        po.close()
     value = total_units / total_dt
-    sample = (f"each step: 1 layer of 1 fork group ({w.n_aux + 1} branches, {w.prefix[0]}-token prefix) "
-              f"of the {w.name} workload, float64 numpy oracle")
+    sample = (f"each step: {po.n} (layer, KV head) units of 1 fork group ({w.n_aux + 1} branches, "
+              f"{w.prefix[0]}-token prefix) of the {w.name} workload, float64 numpy oracle, one per worker "
+              f"process ({po.n} processes, one thread each)")
     return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_dt / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
             "config": {"workload": w.name, "sample": sample},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": po.n, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
@@ -830,6 +912,8 @@ def main():
     ap.add_argument("--n-aux", type=int, default=None,
                     help="config 4 with this many auxiliary branches per group instead of 4")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-workers", type=int, default=None,
+                    help="host worker processes of the oracle baseline (default: one per core)")
     ap.add_argument("--profile-small", action="store_true",
                     help="run the small decode + merge case used for ncu captures and exit")
     ap.add_argument("--profile-wide", action="store_true",
@@ -873,7 +957,7 @@ def main():
         res = run_ours(args, rank, ws, local)
         if rank == 0 and ws == 1 and not args.no_cpu_baseline:
             import torch
-            res["cpu_baseline"] = cpu_baseline(_workload(args), torch.device("cuda", local))
+            res["cpu_baseline"] = cpu_baseline(_workload(args), args.oracle_workers)
     if rank == 0:
         print(json.dumps(res), flush=True)
     if ws > 1:

@@ -47,3 +47,13 @@ def _release_device_memory(request):
                 torch.cuda.empty_cache()
         except ImportError:
             pass
+
+
+@pytest.fixture(scope="session")
+def oracle_jobs():
+    """A pool of float64-oracle worker processes (spawned), shared by the
+    full-size parity tests."""
+    from oracle_jobs import OracleJobs
+    jobs = OracleJobs()
+    yield jobs
+    jobs.close()

@@ -6,6 +6,8 @@ records, per sequence, which (tag, row range) pieces make up its logical
 context (inherited at fork), so the oracle's context for (sequence, layer)
 is rebuilt by re-drawing those pieces -- never read back from the GPU pool.
 """
+import json
+import os
 from collections import OrderedDict
 
 import numpy as np
@@ -16,9 +18,10 @@ from oracle import attention as A
 from oracle import pool as R
 from workloads import kv_rows, queries
 
-# Tolerances of the parity target: element-wise |gpu - oracle| <= 2e-3 + 1e-2 |oracle|
-# for O; |gpu - oracle| <= 1e-4 for the log-sum-exp.
+# Tolerances of the parity target: O within max-abs 2e-3 and max-rel 1e-2 (the
+# relative bound over |oracle| >= REL_FLOOR), the log-sum-exp within 1e-4.
 O_ABS, O_REL, LSE_ABS = 2e-3, 1e-2, 1e-4
+REL_FLOOR = 1e-2
 
 
 class Run:
@@ -152,15 +155,40 @@ class Run:
             assert n == self.ref.seqs[rid].length
 
 
+def _log(what, n, max_abs, max_rel, max_lse):
+    """One JSON line per comparison into $ST_PARITY_LOG, when it is set (the
+    achieved-error figures)."""
+    path = os.environ.get("ST_PARITY_LOG")
+    if not path:
+        return
+    test = os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0]
+    with open(path, "a") as f:
+        f.write(json.dumps({"test": test, "what": what, "n": int(n), "max_abs": max_abs,
+                            "max_rel": max_rel, "max_lse": max_lse}) + "\n")
+
+
 def compare(o_gpu, lse_gpu, o_ref, lse_ref, what=""):
-    """Element-wise check against the oracle; returns (max_abs, max_rel, max_lse)."""
-    o = o_gpu.double().cpu().numpy() if isinstance(o_gpu, torch.Tensor) else o_gpu
-    l = lse_gpu.double().cpu().numpy() if isinstance(lse_gpu, torch.Tensor) else lse_gpu
+    """Element-wise check against the oracle, in two forms:
+    * the stated target read literally: max |gpu - oracle| <= 2e-3 over all
+      O elements, and max |gpu - oracle| / |oracle| <= 1e-2 over the elements
+      with |oracle| >= REL_FLOOR (below it a relative error measures nothing
+      but the rounding of a value near zero);
+    * the allclose reading, |gpu - oracle| <= 2e-3 + 1e-2 |oracle| per
+      element (implied by the first, kept as the survey states it);
+    and |LSE gpu - LSE oracle| <= 1e-4.  Returns (max_abs, max_rel, max_lse)."""
+    o = o_gpu.double().cpu().numpy() if isinstance(o_gpu, torch.Tensor) else np.asarray(o_gpu, np.float64)
+    l = lse_gpu.double().cpu().numpy() if isinstance(lse_gpu, torch.Tensor) else np.asarray(lse_gpu, np.float64)
+    assert o.shape == o_ref.shape and l.shape == lse_ref.shape, what
     assert np.isfinite(o).all() and np.isfinite(l).all(), what
     err = np.abs(o - o_ref)
+    big = np.abs(o_ref) >= REL_FLOOR
+    max_abs = float(err.max(initial=0.0))
+    max_rel = float((err[big] / np.abs(o_ref[big])).max(initial=0.0))
+    max_lse = float(np.abs(l - lse_ref).max(initial=0.0))
+    _log(what, o.size, max_abs, max_rel, max_lse)
     bad = err > O_ABS + O_REL * np.abs(o_ref)
-    lerr = np.abs(l - lse_ref)
-    rel = err / np.maximum(np.abs(o_ref), 1e-30)
-    assert not bad.any(), f"{what}: {bad.sum()} O elements out of tolerance, max abs {err.max():.3e}"
-    assert (lerr <= LSE_ABS).all(), f"{what}: max lse err {lerr.max():.3e}"
-    return float(err.max()), float(rel[np.abs(o_ref) > 1e-3].max(initial=0.0)), float(lerr.max())
+    assert not bad.any(), f"{what}: {bad.sum()} O elements out of tolerance, max abs {max_abs:.3e}"
+    assert max_abs <= O_ABS, f"{what}: max abs O error {max_abs:.3e} > {O_ABS}"
+    assert max_rel <= O_REL, f"{what}: max rel O error {max_rel:.3e} > {O_REL}"
+    assert max_lse <= LSE_ABS, f"{what}: max lse err {max_lse:.3e}"
+    return max_abs, max_rel, max_lse

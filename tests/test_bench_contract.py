@@ -23,7 +23,7 @@ def _check(d, n_gpus):
     assert d["impl"] == "reference" and d["n_gpus"] == n_gpus and d["steps"] == 2 and d["warmup"] == 1
     assert d["value"] > 0 and d["higher_is_better"] is True and d["vs_baseline"] is None
     cb = d["cpu_baseline"]
-    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] == 2 and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     assert d["config"]["workload"] == "tiny_fork_group"
 
@@ -36,7 +36,8 @@ def _env():
 
 def test_reference_arm_one_process():
     r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "1", "--steps", "2",
-                        "--warmup", "1"], cwd=ROOT, env=_env(), capture_output=True, text=True, timeout=300)
+                        "--warmup", "1", "--oracle-workers", "2"], cwd=ROOT, env=_env(), capture_output=True,
+                       text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = _lines(r.stdout)
     assert len(lines) == 1
@@ -50,7 +51,8 @@ def test_reference_arm_two_ranks():
     s.close()
     r = subprocess.run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
                         "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--gpus", "2",
-                        "--impl", "reference", "--config", "1", "--steps", "2", "--warmup", "1"],
+                        "--impl", "reference", "--config", "1", "--steps", "2", "--warmup", "1",
+                        "--oracle-workers", "2"],
                        cwd=ROOT, env=_env(), capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = _lines(r.stdout)

@@ -85,9 +85,7 @@ def test_cfg3_batched_agent_serving(stlib):
     compare(o[0], lse[0], o_ref, l_ref, "cfg3")
 
 
-def test_cfg4_long_trajectory_sampled_layers(stlib):
-    w = get(4)
-    run = _run(w, cache_layers=48)
+def _long_groups(run, w):
     groups = []
     for t in range(w.n_tasks):
         m = run.create()
@@ -98,46 +96,65 @@ def test_cfg4_long_trajectory_sampled_layers(stlib):
             if s:
                 run.append([rid], s, ("suffix", t, b))
         groups.append(br)
+    return groups
+
+
+def _check_every_layer(run, w, groups, q, o, lse, jobs, what):
+    """Every branch of every group on every layer, one (layer, group) oracle
+    job each, spread over the worker processes."""
+    o_cpu, l_cpu, q_cpu = o.cpu(), lse.cpu(), q.cpu()
+    futs, col = [], 0
+    for g in groups:
+        idx = list(range(col, col + len(g)))
+        col += len(g)
+        for layer in range(w.n_layers):
+            futs.append((layer, idx, jobs.decode(w, layer, q_cpu[layer, idx], [run.hist[r] for r in g],
+                                                  run.sizes)))
+    for layer, idx, f in futs:
+        o_ref, l_ref = f.get()
+        compare(o_cpu[layer, idx], l_cpu[layer, idx], o_ref, l_ref, f"{what} layer {layer} rows {idx[0]}..")
+
+
+def test_cfg4_long_trajectory_every_layer(stlib, oracle_jobs):
+    """The long-trajectory workload at full size (4 groups x 131072-token
+    prefixes, 32 layers): every branch checked on every layer."""
+    w = get(4)
+    run = _run(w, cache_layers=48)
+    groups = _long_groups(run, w)
     rids = [r for g in groups for r in g]
     run.append(rids, 1, ("step",))
     q, o, lse = run.decode(rids, ("q",))
     run.pool.sync()
     run.check_tables()
-    for layer in (0, w.n_layers - 1):
-        o_ref, l_ref = run.oracle_decode(rids, q, layer)
-        compare(o[layer], lse[layer], o_ref, l_ref, f"cfg4 layer {layer}")
+    _check_every_layer(run, w, groups, q, o, lse, oracle_jobs, "cfg4")
 
 
 @pytest.mark.parametrize("n_aux", [8, 16])
-def test_cfg4_long_trajectory_wide_sampled_layers(stlib, n_aux):
+def test_cfg4_long_trajectory_wide_every_layer(stlib, oracle_jobs, n_aux):
     """The long-trajectory workload at full size with 9 branches per group (72
     stacked rows: one wide tile per group) and 17 (136 rows: two wide subgroups
     whose second read of each prefix page comes from L2), as `bench.py --n-aux`
-    times it."""
+    times it; every branch on every layer."""
     from workloads.configs import long_with_branches
     w = long_with_branches(n_aux)
     run = _run(w, cache_layers=48)
-    groups = []
-    for t in range(w.n_tasks):
-        m = run.create()
-        _prefix(run, m, w.prefix[t], ("prefix", t))
-        aux = run.fork(m, w.n_aux)
-        br = [m] + aux
-        for b, (rid, s) in enumerate(zip(br, w.suffix[t])):
-            if s:
-                run.append([rid], s, ("suffix", t, b))
-        groups.append(br)
+    groups = _long_groups(run, w)
     rids = [r for g in groups for r in g]
     run.append(rids, 1, ("step",))
     q, o, lse = run.decode(rids, ("q",))
     run.pool.sync()
     run.check_tables()
-    for layer in (0, w.n_layers - 1):
-        o_ref, l_ref = run.oracle_decode(rids, q, layer)
-        compare(o[layer], lse[layer], o_ref, l_ref, f"{w.name} layer {layer}")
+    _check_every_layer(run, w, groups, q, o, lse, oracle_jobs, w.name)
 
 
-def test_cfg5_full_cycle_sampled(stlib):
+def test_cfg5_full_cycle(stlib, oracle_jobs):
+    """The full cycle (8 tasks x 5 turns of fork, 512 append + decode steps,
+    merge of 2048 thought rows, release; 64 unforked sequences per turn).
+    Tables, refcounts and the free list are compared after every turn; O and
+    LSE of all 104 branches at steps 1, 64, 128, ..., 512 of every turn (each
+    check on its own layer); every row of turn 1 / task 0's merge, and for the
+    other merges 1 row in 16: the first and last row of each 64-row work item
+    plus a seeded sample."""
     w = get(5)
     run = _run(w, cache_layers=32)
     mains = []
@@ -146,7 +163,11 @@ def test_cfg5_full_cycle_sampled(stlib):
         _prefix(run, m, w.prefix[t], ("prefix", t))
         mains.append(m)
     rng = np.random.default_rng(5)
-    check_steps = {0, 255, w.steps - 1}
+    check_steps = [0] + list(range(63, w.steps, 64))   # steps 1, 64, 128, ..., 512 counted from 1
+    T = w.merge_tokens
+    chunk = 256 // w.group                               # thought rows per merge work item
+    futs = []
+    n_check = 0
     for turn in range(w.turns):
         singles = [run.create() for _ in range(w.singletons)]
         for i in range(0, w.singletons, 8):
@@ -157,19 +178,32 @@ def test_cfg5_full_cycle_sampled(stlib):
             run.append(rids, 1, ("step", turn, step))
             q, o, lse = run.decode(rids, ("q", turn, step))
             if step in check_steps:
-                layer = (7 * turn + step) % w.n_layers
-                sample = groups[turn % w.n_tasks] + singles[:2]
-                idx = [rids.index(r) for r in sample]
-                o_ref, l_ref = run.oracle_decode(sample, q[:, idx], layer)
-                compare(o[layer][idx], lse[layer][idx], o_ref, l_ref, f"cfg5 turn {turn} step {step}")
+                layer = (5 * n_check + 3) % w.n_layers
+                n_check += 1
+                o_c, l_c, q_c = o[layer].cpu(), lse[layer].cpu(), q[layer].cpu()
+                for b0 in range(0, len(rids), 26):
+                    sl = slice(b0, b0 + 26)
+                    f = oracle_jobs.decode(w, layer, q_c[sl], [list(run.hist[r]) for r in rids[sl]],
+                                           dict(run.sizes))
+                    futs.append((f"cfg5 turn {turn} step {step + 1} layer {layer} branches {b0}..",
+                                 o_c[sl], l_c[sl], f))
         for t, m in enumerate(mains):
-            qm, om, lm, L0 = run.merge(m, w.merge_tokens, ("merge", turn, t))
-            if t == turn % w.n_tasks:
-                layer = (3 * turn + 1) % w.n_layers
-                rows = sorted({0, 1, 63, 64, w.merge_tokens - 1, *rng.integers(0, w.merge_tokens, 6).tolist()})
-                k, v = run.context(m, layer)
-                o_ref, l_ref = A.merge_prefill(qm[layer].cpu(), k, v, L0, rows=rows)
-                compare(om[layer][rows], lm[layer][rows], o_ref, l_ref, f"cfg5 merge turn {turn}")
+            pieces = list(run.hist[m])
+            qm, om, lm, L0 = run.merge(m, T, ("merge", turn, t))
+            layer = (11 * turn + 3 * t + 1) % w.n_layers
+            if turn == 0 and t == 0:
+                rows = list(range(T))
+            else:
+                edge = {r for c0 in range(0, T, chunk) for r in (c0, min(c0 + chunk, T) - 1)}
+                rest = sorted(set(range(T)) - edge)
+                rows = sorted(edge | set(rng.choice(rest, T // 16 - len(edge), replace=False).tolist()))
+            pieces = pieces + [(("merge", turn, t), 0, T)]
+            q_c, o_c, l_c = qm[layer].cpu(), om[layer].cpu(), lm[layer].cpu()
+            for r0 in range(0, len(rows), 128):
+                part = rows[r0:r0 + 128]
+                f = oracle_jobs.merge(w, layer, q_c, pieces, dict(run.sizes), L0, part)
+                futs.append((f"cfg5 merge turn {turn} task {t} layer {layer} rows {part[0]}..{part[-1]}",
+                             o_c[part], l_c[part], f))
         for g in groups:
             for a in g[1:]:
                 run.release(a)
@@ -177,6 +211,9 @@ def test_cfg5_full_cycle_sampled(stlib):
             run.release(s)
         run.pool.sync()
         run.check_tables()
+    for what, o_g, l_g, f in futs:
+        o_ref, l_ref = f.get()
+        compare(o_g, l_g, o_ref, l_ref, what)
 
 
 # ---- edge cases on small shapes -------------------------------------------
