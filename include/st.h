@@ -296,28 +296,36 @@ ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, in
  * calls that overlap on the GPU (different streams without ordering) race.
  *
  * geom:        pool geometry (n_layers, n_q_heads, n_kv_heads, head_dim,
- *              page_size = 16, n_blocks); other fields are ignored.
+ *              page_size = 16, n_blocks); of the flags only ST_FLAG_HOLD_LOADS
+ *              is honoured; other fields are ignored.
  * k_pool/v_pool: device bf16 [n_layers][n_blocks][n_kv_heads][16][head_dim]
  *              (the st_pool_create layout), 16-byte aligned.
  * page_table:  HOST int32 [n_br][table_stride], each branch's physical page
- *              ids in logical order; ids must lie in [0, n_blocks).
+ *              ids in logical order; the first ceil(seq_len / 16) of each
+ *              row must lie in [0, n_blocks) (checked; ST_ERR_INVALID).
  * seq_len:     HOST int32 [n_br], tokens in each branch's context (>= 1,
  *              ceil(len / 16) <= table_stride).
  * q, o, lse:   as st_decode_attn, on the current device.
+ * status:      DEVICE int32 [1], caller-owned.  The call clears it on
+ *              `stream` before its kernels run; once the stream has passed
+ *              the call it holds ST_OK, ST_ERR_TIMEOUT (a device-side wait ran
+ *              past its limit: o and lse are then undefined) or
+ *              ST_ERR_INVALID (a device-side bounds check fired).  The return
+ *              value covers only what the host can see when the call returns.
  * Branches whose tables start on the same physical page are treated as one
- * fork group: their common full pages are read once for the group.
+ * fork group: their common full pages are read once for the group (groups
+ * of more than 48 / G branches are split into several).
  * Returns ST_ERR_INVALID for bad arguments or n_br > ST_NOALLOC_MAX_BRANCHES,
  * and ST_ERR_OOM when the call needs more than the static scratch:
- *   256-byte-rounded 37 KiB plan + 4*n_br*table_stride
+ *   36.25 KiB of plan + 4*n_br*table_stride (rounded up to 256 bytes)
  *   + 4*n_layers*n_br*n_q_heads*16*(head_dim + 1) bytes > 16 MiB.
- * The work runs on `stream`; device-side bounds checks skip a bad page id
- * (it reads as zeros) without reporting it. */
+ * The work runs on `stream`. */
 #define ST_NOALLOC_SCRATCH_BYTES (16u << 20)
 #define ST_NOALLOC_MAX_BRANCHES 64
 ST_API st_status st_decode_attn_noalloc(const st_config* geom, const void* k_pool, const void* v_pool,
                                         const int32_t* page_table, int table_stride,
                                         const int32_t* seq_len, int n_br, const void* q, float* o,
-                                        float* lse, void* stream);
+                                        float* lse, int32_t* status, void* stream);
 
 ST_API const char* st_status_str(st_status s);
 ST_API const char* st_last_error(st_pool* pool);

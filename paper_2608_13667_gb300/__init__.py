@@ -91,7 +91,7 @@ def lib():
         "st_profile_enable": (I, [P, I]),
         "st_profile_read": (I, [P, ctypes.POINTER(StKernelStat), I, ctypes.POINTER(I)]),
         "st_harvest": (I, [VP, I, VP, I, ctypes.c_int32, ctypes.c_int32, I, VP, VP, VP, VP, VP]),
-        "st_decode_attn_noalloc": (I, [ctypes.POINTER(StConfig), VP, VP, i32p, I, i32p, I, VP, VP, VP, VP]),
+        "st_decode_attn_noalloc": (I, [ctypes.POINTER(StConfig), VP, VP, i32p, I, i32p, I, VP, VP, VP, VP, VP]),
         "st_status_str": (ctypes.c_char_p, [I]),
         "st_last_error": (ctypes.c_char_p, [P]),
     }
@@ -435,11 +435,13 @@ def st_harvest(streams, lens, open_id, close_id, cap=5, stream=None):
     return out_ids[:T], out_src[:T], atoms
 
 
-def st_decode_attn_noalloc(geom, k_pool, v_pool, page_tables, seq_len, q, o, lse, stream=None):
+def st_decode_attn_noalloc(geom, k_pool, v_pool, page_tables, seq_len, q, o, lse, status=None, stream=None):
     """Allocation-free decode (see include/st.h): geom is a StConfig, k_pool/v_pool
     the bf16 KV tensors, page_tables a list of per-branch page-id lists (host),
     seq_len per-branch token counts, q/o/lse device tensors as for
-    st_decode_attn.  Returns the status code."""
+    st_decode_attn, status a device int32 tensor of one element (made here if
+    None) that holds the device-side outcome once the stream has passed the
+    call.  Returns (status code of the call, status tensor)."""
     import torch
     n_br = len(seq_len)
     stride = max(1, max(len(t) for t in page_tables))
@@ -448,9 +450,13 @@ def st_decode_attn_noalloc(geom, k_pool, v_pool, page_tables, seq_len, q, o, lse
         for j, b in enumerate(t):
             table[i * stride + j] = b
     lens = (ctypes.c_int32 * n_br)(*[int(x) for x in seq_len])
+    if status is None:
+        status = torch.empty(1, dtype=torch.int32, device=q.device)
     if stream is None:
         stream = torch.cuda.current_stream(q.device)
-    return lib().st_decode_attn_noalloc(ctypes.byref(geom), ctypes.c_void_p(k_pool.data_ptr()),
-                                        ctypes.c_void_p(v_pool.data_ptr()), table, stride, lens, n_br,
-                                        ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(o.data_ptr()),
-                                        ctypes.c_void_p(lse.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+    st = lib().st_decode_attn_noalloc(ctypes.byref(geom), ctypes.c_void_p(k_pool.data_ptr()),
+                                      ctypes.c_void_p(v_pool.data_ptr()), table, stride, lens, n_br,
+                                      ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(o.data_ptr()),
+                                      ctypes.c_void_p(lse.data_ptr()), ctypes.c_void_p(status.data_ptr()),
+                                      ctypes.c_void_p(stream.cuda_stream))
+    return st, status

@@ -14,13 +14,17 @@
 // The array is ST_NOALLOC_SCRATCH_BYTES (16 MiB) per device and stays
 // allocated on every GPU that loads the library until the process exits.
 // Every call reuses it: calls that overlap on the GPU (different streams
-// without ordering) race on it.  Nothing in it needs to start at zero except
-// the status word, which each call's plan upload clears.
+// without ordering) race on it.  Nothing in it needs to start at zero: the
+// plan and the page-table copy are uploaded whole by each call, and every
+// partial slot the combine reads is written by that call's decode.  Device
+// errors (a wait that ran out, a page id out of range) go to the caller's
+// status word, which the call clears first.
 #include <cudaTypedefs.h>
 
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 
 #include "../../include/st.h"
 #include "kernels.cuh"
@@ -38,41 +42,51 @@ constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
-// Device address of the array, per device.  In host code the array's name is
-// only a host-side stand-in, so the address comes from cudaGetSymbolAddress,
-// taken once per device with that device current.
-void* g_scratch_dev[kMaxDevices] = {};
-int g_ctas_per_sm[kMaxDevices][2] = {};  // [dev][head_dim == 128]
-int g_sms[kMaxDevices] = {};
+// Per device, set up once (std::call_once, so two host threads making their
+// first call together are safe): the device address of the array -- in host
+// code the array's name is only a host-side stand-in, so the address comes
+// from cudaGetSymbolAddress with that device current -- and the launch
+// geometry the planner sizes runs by.
+struct DeviceSetup {
+  std::once_flag once;
+  st_status status = ST_ERR_CUDA;
+  void* scratch = nullptr;
+  int sms = 0;
+  int ctas_per_sm[2] = {};  // [head_dim == 128]
+};
+DeviceSetup g_dev[kMaxDevices];
 
 size_t up256(size_t x) { return (x + 255) / 256 * 256; }
 
-st_status setup_device(int dev) {
-  if (dev < 0 || dev >= kMaxDevices) return ST_ERR_INVALID;
-  if (g_scratch_dev[dev]) return ST_OK;
-  void* p = nullptr;
-  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return ST_ERR_CUDA;
-  int sms = 0;
-  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return ST_ERR_CUDA;
-  const int per_sm = decode_tc_ctas_per_sm(128);
-  const int per_sm64 = decode_tc_ctas_per_sm(64);
-  if (per_sm < 1 || per_sm64 < 1) return ST_ERR_CUDA;
-  g_sms[dev] = sms;
-  g_ctas_per_sm[dev][1] = per_sm;
-  g_ctas_per_sm[dev][0] = per_sm64;
-  g_scratch_dev[dev] = p;
-  return ST_OK;
+const DeviceSetup* setup_device(int dev) {
+  if (dev < 0 || dev >= kMaxDevices) return nullptr;
+  DeviceSetup& d = g_dev[dev];
+  std::call_once(d.once, [&] {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return;
+    if (cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return;
+    d.ctas_per_sm[1] = decode_tc_ctas_per_sm(128);
+    d.ctas_per_sm[0] = decode_tc_ctas_per_sm(64);
+    if (d.ctas_per_sm[0] < 1 || d.ctas_per_sm[1] < 1) return;
+    d.scratch = p;
+    d.status = ST_OK;
+  });
+  return &d;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 lookup_encode() {
+  PFN_cuTensorMapEncodeTiled_v12000 f = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&f), 12000,
+                                       cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess)
+    return nullptr;
+  return f;
 }
 
 bool encode_map(CUtensorMap* map, const void* base, const st_config& c) {
-  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-  if (!encode) {
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&encode),
-                                         12000, cudaEnableDefault, &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return false;
-  }
+  static const PFN_cuTensorMapEncodeTiled_v12000 encode = lookup_encode();  // initialised once, thread-safe
+  if (!encode) return false;
   const int D = c.head_dim;
   cuuint64_t dims[4] = {64, (cuuint64_t)(D / 64), (cuuint64_t)kPageTokens * c.n_kv_heads,
                         (cuuint64_t)c.n_layers * (cuuint64_t)c.n_blocks};
@@ -92,7 +106,6 @@ void split_even(int32_t n, int32_t k, int32_t c, int32_t* begin, int32_t* count)
 
 // Host-side plan, kept on the stack (fixed maximum sizes).
 struct NoallocPlan {
-  int32_t status[16];
   AttnItem items[kMaxItems];
   int32_t members[kMaxItems];
   int32_t n_splits[kMaxBranches];
@@ -103,19 +116,27 @@ struct NoallocPlan {
 extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const void* k_pool,
                                                    const void* v_pool, const int32_t* page_table,
                                                    int table_stride, const int32_t* seq_len, int n_br,
-                                                   const void* q, float* o, float* lse, void* stream) {
-  if (!geom || !k_pool || !v_pool || !page_table || !seq_len || !q || !o || !lse) return ST_ERR_INVALID;
+                                                   const void* q, float* o, float* lse, int32_t* status,
+                                                   void* stream) {
+  if (!geom || !k_pool || !v_pool || !page_table || !seq_len || !q || !o || !lse || !status)
+    return ST_ERR_INVALID;
   const st_config& c = *geom;
   if (c.n_layers < 1 || c.n_kv_heads < 1 || c.n_q_heads % c.n_kv_heads != 0 ||
       c.n_q_heads / c.n_kv_heads > kMaxRows || (c.head_dim != 64 && c.head_dim != 128) ||
       c.page_size != kPageTokens || c.n_blocks < 1 || (int64_t)c.n_layers * c.n_blocks >= INT32_MAX)
     return ST_ERR_INVALID;
   if (n_br < 1 || n_br > kMaxBranches || table_stride < 1) return ST_ERR_INVALID;
-  if (((uintptr_t)k_pool | (uintptr_t)v_pool | (uintptr_t)q | (uintptr_t)o) % 16 != 0) return ST_ERR_INVALID;
+  if (((uintptr_t)k_pool | (uintptr_t)v_pool | (uintptr_t)q | (uintptr_t)o) % 16 != 0 ||
+      ((uintptr_t)lse | (uintptr_t)status) % 4 != 0)
+    return ST_ERR_INVALID;
   const int G = c.n_q_heads / c.n_kv_heads;
-  for (int i = 0; i < n_br; ++i)
+  for (int i = 0; i < n_br; ++i) {
     if (seq_len[i] < 1 || (int64_t)(seq_len[i] + kPageTokens - 1) / kPageTokens > table_stride)
       return ST_ERR_INVALID;
+    const int32_t* t = page_table + (size_t)i * table_stride;
+    for (int32_t p = 0; p < (seq_len[i] + kPageTokens - 1) / kPageTokens; ++p)
+      if (t[p] < 0 || t[p] >= c.n_blocks) return ST_ERR_INVALID;
+  }
 
   // scratch layout and its limit
   const size_t off_plan = 0;
@@ -128,13 +149,13 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
 
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return ST_ERR_CUDA;
-  st_status st = setup_device(dev);
-  if (st != ST_OK) return st;
-  unsigned char* scratch = static_cast<unsigned char*>(g_scratch_dev[dev]);
+  const DeviceSetup* ds = setup_device(dev);
+  if (!ds) return ST_ERR_INVALID;
+  if (ds->status != ST_OK) return ds->status;
+  unsigned char* scratch = static_cast<unsigned char*>(ds->scratch);
 
   // ---- plan: fork groups = branches whose tables start on the same page ----
   NoallocPlan plan;
-  std::memset(plan.status, 0, sizeof plan.status);
   int32_t shared[kMaxBranches] = {};
   int32_t n_items = 0, n_members = 0;
   int64_t total_pages = 0;
@@ -179,7 +200,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
     plan.n_splits[i] = 0;
   }
   const int64_t units = total_pages * c.n_kv_heads * c.n_layers;
-  const int64_t target = (int64_t)32 * g_sms[dev] * g_ctas_per_sm[dev][c.head_dim == 128];
+  const int64_t target = (int64_t)32 * ds->sms * ds->ctas_per_sm[c.head_dim == 128];
   int64_t chunk = std::max<int64_t>(16, ((units + target - 1) / target + 3) / 4 * 4);
   for (int gi = 0; gi < n_groups; ++gi) {
     const Grp& g = groups[gi];
@@ -212,7 +233,8 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   if (!encode_map(&kmap, k_pool, c) || !encode_map(&vmap, v_pool, c)) return ST_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // pageable host sources: the copies have consumed them when these calls return
-  if (cudaMemcpyAsync(scratch + off_plan, &plan, sizeof plan, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+  if (cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess ||
+      cudaMemcpyAsync(scratch + off_plan, &plan, sizeof plan, cudaMemcpyHostToDevice, s) != cudaSuccess ||
       cudaMemcpyAsync(scratch + off_table, page_table, (size_t)n_br * table_stride * sizeof(int32_t),
                       cudaMemcpyHostToDevice, s) != cudaSuccess)
     return ST_ERR_CUDA;
@@ -225,7 +247,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   ap.table = reinterpret_cast<const int32_t*>(scratch + off_table);
   ap.items = dplan->items;
   ap.members = dplan->members;
-  ap.status = dplan->status;
+  ap.status = status;
   ap.n_blocks = c.n_blocks;
   ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c.head_dim));
   ap.n_rows_q = n_br;
@@ -235,6 +257,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
   ap.L = c.n_layers;
   ap.max_pages = table_stride;
   ap.max_splits = kSplitStride;
+  ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
   if (launch_decode_tc(kmap, vmap, ap, nullptr, n_items, c.head_dim, false, s) != cudaSuccess) return ST_ERR_CUDA;
   CombineParams cp{};
   cp.part_o = ap.out_o;
