@@ -362,6 +362,19 @@ def run_ours(args, rank, ws, local):
                               "overlapping the neighbouring steps' compute"},
         }
     pool.close()
+    if rank == 0:
+        # the tensor-bound half of the path: the merge prefill, timed alone on a
+        # fixed case in the same run
+        mg = _merge_case(3, dev)
+        peaks, src = _peaks()
+        res["merge"] = {
+            "kernel": "merge_prefill", "workload": MERGE_CASE,
+            "ms": mg["merge_ms"], "launches": mg["merge_launches"],
+            "roofline": {"bound": "tensor", "achieved": mg["merge_tflops"], "peak": peaks["bf16_tflops"],
+                         "peak_source": src + " (bf16 burst: the kernel is timed alone)", "unit": "TFLOP/s",
+                         "frac": mg["merge_tflops"] / peaks["bf16_tflops"],
+                         "flops": "algorithmic: 4 D x causal keys x q heads x layers; P V runs for both bf16 "
+                                  "terms of P, so the tensor cores execute 1.5x this"}}
     return res
 
 
@@ -399,7 +412,11 @@ def run_profile_small():
                       "decode_gbs": d["bytes"] / d["total_ms"] / 1e6, **mg}))
 
 
-def _merge_case(n_merges=3):
+MERGE_CASE = ("2048 thought rows merged onto a 16896-token main context (the full cycle's first merge), "
+              "32 q / 8 kv heads, D 128, 4 layers")
+
+
+def _merge_case(n_merges=3, dev=None):
     """Merges of 2048 thought rows onto a 16896-token main context (32 q / 8 kv
     heads, D 128, 4 layers): main is forked n_merges times and each fork takes
     one merge, so every launch does the same work.  Returns the CUDA-event
@@ -408,7 +425,7 @@ def _merge_case(n_merges=3):
     import torch
     import paper_2608_13667_gb300 as st
     from workloads import get, kv_rows, queries
-    dev = torch.device("cuda", 0)
+    dev = dev or torch.device("cuda", 0)
     st.build()
     w5 = dataclasses.replace(get(5), n_layers=4)
     p5 = st.Pool(n_layers=4, n_q_heads=w5.n_q_heads, n_kv_heads=w5.n_kv_heads, head_dim=w5.head_dim,
@@ -432,7 +449,7 @@ def _merge_case(n_merges=3):
             best = mg
     p5.close()
     return {"merge_ms": best["total_ms"], "merge_tflops": best["flops"] / best["total_ms"] / 1e9,
-            "merges": n_merges}
+            "merges": n_merges, "merge_launches": n_merges}
 
 
 def run_profile_wide():
