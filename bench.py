@@ -452,10 +452,11 @@ def _merge_case(n_merges=3, dev=None):
             "merges": n_merges, "merge_launches": n_merges}
 
 
-def run_profile_wide():
+def run_profile_wide(n_aux=None):
     """The wide decode tile on a small case for ncu captures: the long-trajectory
-    decode with 9 branches per group (72 stacked rows) and 4 layers instead of 32,
-    three decode steps.  Prints the CUDA-event timing of the last one."""
+    decode with 9 branches per group (72 stacked rows; another count with
+    --n-aux, e.g. 16 for the paired tile's 136 rows) and 4 layers instead of
+    32, three decode steps.  Prints the CUDA-event timing of the last one."""
     import dataclasses
     import torch
     import paper_2608_13667_gb300 as st
@@ -463,7 +464,7 @@ def run_profile_wide():
     from workloads.configs import long_with_branches
     dev = torch.device("cuda", 0)
     st.build()
-    w = dataclasses.replace(long_with_branches(8), n_layers=4)
+    w = dataclasses.replace(long_with_branches(8 if n_aux is None else n_aux), n_layers=4)
     pool, br = build_long_workload(w, dev)
     n = len(br)
     o = torch.empty((w.n_layers, n, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
@@ -962,7 +963,7 @@ def main():
         run_turn()
         return
     if args.profile_wide:
-        run_profile_wide()
+        run_profile_wide(args.n_aux)
         return
     if args.cycle:
         run_cycle()

@@ -71,6 +71,9 @@ struct AttnItem {
 constexpr int32_t kItemReread = 1;
 // more than 48 stacked rows: the M = 128 tile
 constexpr int32_t kItemWide = 2;
+// more than 128 stacked rows: two M = 128 tiles of one CTA sharing every K/V
+// stage (the merge's paired tile, merge_tc.cu)
+constexpr int32_t kItemPair = 4;
 
 // One CTA of a batched merge / prefill: rows [row_base, row_base + 256) of
 // one sequence's stacked (new row, head) rows.
@@ -174,6 +177,11 @@ cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, c
 // batch of n_items work items (p.mitems), p.q -> p.out_o, p.out_lse.
 cudaError_t launch_merge_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int n_items,
                             int D, cudaStream_t s);
+// Decode partials of fork groups of 129 to 256 stacked rows on the same
+// paired tile (one CTA per item x KV head x layer, items from p.item_base on,
+// launched as a programmatic dependent like the other decode kernels).
+cudaError_t launch_decode_pair(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,
+                               const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s);
 // CTAs of the tcgen05 decode kernel resident per SM (0 on error).
 int decode_tc_ctas_per_sm(int D);
 

@@ -101,10 +101,10 @@ struct PairCfg {
   static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
 
-template <int D>
+template <int D, bool kDecode>
 __global__ void __launch_bounds__(kThreads, 1)
     merge_pair_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                      const AttnParams p) {
+                      const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
   using C = PairCfg<D>;
   constexpr int kKS = C::kKStages, kVS = C::kVStages;
   extern __shared__ uint8_t smem_raw[];
@@ -127,21 +127,45 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int layer = blockIdx.z;
   const int G = p.G;
 
-  // one merge: its row tiles, the last ones (most keys) first; a batch: one
-  // work item per CTA (the host orders those longest first)
-  int slot = p.slot, L0 = p.L0, T = p.T, q_row0 = 0, row_base = (gridDim.x - 1 - blockIdx.x) * 2 * kTileRows;
-  if (p.mitems) {
-    const MergeItem mi = p.mitems[blockIdx.x];
-    slot = mi.slot;
-    L0 = mi.L0;
-    T = mi.T;
-    q_row0 = mi.q_row0;
-    row_base = mi.row_base;
+  // Decode: launched as a programmatic dependent of the kernel before it in
+  // the stream; the tensor-memory allocation touches no global memory, every
+  // global access comes after the wait.
+  if constexpr (kDecode) {
+    if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
+    griddep_wait();
+    griddep_launch_dependents();
   }
-  const int n_rows = min(2 * kTileRows, T * G - row_base);
-  const int t_last = (row_base + n_rows - 1) / G;
-  const int n_pages = (L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
-  const int n_valid_keys = L0 + T;
+  // one merge: its row tiles, the last ones (most keys) first; a batch: one
+  // work item per CTA (the host orders those longest first); a decode: one
+  // run of pages of a fork group (at most 256 stacked rows) per CTA, every
+  // row over all of the run's keys
+  int slot = p.slot, L0 = p.L0, T = p.T, q_row0 = 0, row_base = (gridDim.x - 1 - blockIdx.x) * 2 * kTileRows;
+  int page_begin = 0, n_rows, n_pages, n_valid_keys;
+  AttnItem item{};
+  const int32_t* members = nullptr;
+  if constexpr (kDecode) {
+    members = p.members ? p.members : inl.members;
+    item = p.items ? p.items[p.item_base + blockIdx.x] : inl.items[p.item_base + blockIdx.x];
+    slot = item.slot;
+    page_begin = item.page_begin;
+    row_base = 0;
+    n_rows = min(2 * kTileRows, item.n_members * G);
+    n_pages = item.n_pages;
+    n_valid_keys = item.n_tokens;
+  } else {
+    if (p.mitems) {
+      const MergeItem mi = p.mitems[blockIdx.x];
+      slot = mi.slot;
+      L0 = mi.L0;
+      T = mi.T;
+      q_row0 = mi.q_row0;
+      row_base = mi.row_base;
+    }
+    n_rows = min(2 * kTileRows, T * G - row_base);
+    const int t_last = (row_base + n_rows - 1) / G;
+    n_pages = (L0 + t_last + 1 + kPageTokens - 1) / kPageTokens;
+    n_valid_keys = L0 + T;
+  }
   const int n_tiles = (n_pages + kPagesPerStage - 1) / kPagesPerStage;
 
   if (threadIdx.x == 0) {
@@ -162,7 +186,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_ready, kSoftThreads);
     fence_mbar_init();
   }
-  if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
+  if (!kDecode && warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
@@ -178,9 +202,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_st = is_k ? kKS : kVS;
     uint8_t* ring = base + (is_k ? C::kKOff : C::kVOff);
     if (lane == 0) prefetch_tensormap(map);
-    // every CTA of one (layer, KV head) walks the same pages: keep them in L2
-    const uint64_t policy = l2_policy_evict_last();
-    const int32_t* ids = p.table + (int64_t)slot * p.max_pages;
+    // merge: every CTA of one (layer, KV head) walks the same pages, keep them
+    // in L2; decode: a page is streamed once, unless a sibling subgroup's CTA
+    // reads it too or the whole launch fits in L2
+    const uint64_t policy = !kDecode ? l2_policy_evict_last()
+                            : (p.keep_l2 || (item.flags & kItemReread)) ? l2_policy_evict_normal()
+                                                                         : l2_policy_evict_first();
+    const int32_t* ids = p.table + (int64_t)slot * p.max_pages + page_begin;
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
     int nxt = 32 + lane < n_pages ? ids[32 + lane] : 0;
@@ -324,11 +352,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   int qrow = 0, head = 0;
   if (valid) {
     const int gr = tile_row0 + r;
-    qrow = gr / G;
+    qrow = kDecode ? members[item.member_base + gr / G] : gr / G;
     head = kvh * G + gr % G;
   }
-  const int limit = valid ? L0 + qrow + 1 : n_valid_keys;
-  const int min_limit = L0 + tile_row0 / G + 1;  // the tile's first row sees the fewest keys
+  // causal limit of this row (a decode row sees the whole run)
+  const int limit = kDecode ? n_valid_keys : valid ? L0 + qrow + 1 : n_valid_keys;
+  const int min_limit = kDecode ? n_valid_keys : L0 + tile_row0 / G + 1;  // the tile's first row sees the fewest keys
   const int64_t io_row = (int64_t)layer * p.n_rows_q + q_row0 + qrow;  // this row in Q / O / LSE
   {
     const uint4* src = reinterpret_cast<const uint4*>(p.q + (io_row * p.Hq + head) * D);
@@ -457,7 +486,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after_sync();
   if (ok) {
     const float inv = 1.f / l;
-    float* dst = valid ? p.out_o + (io_row * p.Hq + head) * D : nullptr;
+    // merge: the row's O and LSE; decode: its split-KV partial
+    const int64_t out_idx = kDecode ? (io_row * p.Hq + head) * p.max_splits + item.split : io_row * p.Hq + head;
+    float* dst = valid ? p.out_o + out_idx * D : nullptr;
 #pragma unroll 1
     for (int k = 0; k < D / 32; ++k) {
       float o[32];
@@ -469,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               make_float4(o[i] * inv, o[i + 1] * inv, o[i + 2] * inv, o[i + 3] * inv);
       }
     }
-    if (valid) p.out_lse[io_row * p.Hq + head] = (m_used + log2f(l)) * kLn2;
+    if (valid) p.out_lse[out_idx] = (m_used + log2f(l)) * kLn2;
   } else if (lane == 0) {
     atomicCAS(p.status, 0, kDevTimeout);
   }
@@ -477,9 +508,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   named_barrier_sync(1, kSoftThreads + 32);
 }
 
-template <int D>
-cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p, int n_ctas,
-                          cudaStream_t s) {
+template <int D, bool kDecode>
+cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
+                          const InlineDecodePlan& inl, int n_ctas, cudaStream_t s) {
   using C = PairCfg<D>;
   // the shared-memory opt-in is a per-device function attribute
   static bool configured[64] = {};
@@ -488,14 +519,19 @@ cudaError_t launch_pair_t(const CUtensorMap& km, const CUtensorMap& vm, const At
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    e = cudaFuncSetAttribute(merge_pair_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    e = cudaFuncSetAttribute(merge_pair_kernel<D, kDecode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  merge_pair_kernel<D><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p);
+  if constexpr (kDecode)
+    return launch_chained(merge_pair_kernel<D, true>, grid, dim3(kThreads), C::kSmemBytes, s, km, vm, p, inl);
+  merge_pair_kernel<D, false><<<grid, kThreads, C::kSmemBytes, s>>>(km, vm, p, inl);
   return cudaGetLastError();
 }
+
+const InlineDecodePlan kNoInline{};
 
 }  // namespace
 
@@ -504,8 +540,17 @@ cudaError_t launch_merge_tc(const CUtensorMap& km, const CUtensorMap& vm, const 
   // one merge: ceil(T G / 256) row tiles; a batch: its work items
   const int n_ctas = p.mitems ? n_items : (p.T * p.G + 2 * kTileRows - 1) / (2 * kTileRows);
   if (n_ctas <= 0) return cudaSuccess;
-  if (D == 128) return launch_pair_t<128>(km, vm, p, n_ctas, s);
-  if (D == 64) return launch_pair_t<64>(km, vm, p, n_ctas, s);
+  if (D == 128) return launch_pair_t<128, false>(km, vm, p, kNoInline, n_ctas, s);
+  if (D == 64) return launch_pair_t<64, false>(km, vm, p, kNoInline, n_ctas, s);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_decode_pair(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
+                               const InlineDecodePlan* inl, int n_items, int D, cudaStream_t s) {
+  const InlineDecodePlan& ip = inl ? *inl : kNoInline;
+  if (n_items <= 0) return cudaSuccess;
+  if (D == 128) return launch_pair_t<128, true>(km, vm, p, ip, n_items, s);
+  if (D == 64) return launch_pair_t<64, true>(km, vm, p, ip, n_items, s);
   return cudaErrorInvalidValue;
 }
 

@@ -35,7 +35,8 @@ namespace {
 constexpr int kStageSlots = 8;
 constexpr size_t kStageSlotBytes = 2u << 20;  // 2 MiB per plan
 constexpr int kMaxAttnRows = 48;              // stacked query rows of the narrow decode tile
-constexpr int kMaxWideRows = 128;             // ... and of the wide one
+constexpr int kMaxWideRows = 128;             // ... of the wide one
+constexpr int kMaxPairRows = 256;             // ... and of the paired tile
 
 enum KernelId { kKTable = 0, kKAppend, kKDecode, kKCombine, kKMerge, kNumKernels };
 const char* const kKernelNames[kNumKernels] = {"table_update", "append_kv", "decode_partial",
@@ -117,6 +118,26 @@ struct Plan {
   }
 };
 
+// The decode work decomposition of one st_decode_attn call (host only; the
+// same plan st_decode_plan reports), filled by plan_decode below.
+struct DecodePlan {
+  std::vector<AttnItem> items;
+  std::vector<int32_t> members;   // the call's branch index of each item's members
+  std::vector<int32_t> n_splits;  // partials per branch
+  // algorithmic, whole launch: every KV page once per fork family and layer
+  // (shared pages once for the family, own pages once for their branch) and
+  // the queries
+  double bytes = 0, flops = 0;
+  double reread_bytes = 0;        // second and later reads of a split family's pages
+  double part_bytes = 0;          // the split-KV partials (written here, read by the combine)
+  // scratch of the planner, kept between calls so that a decode step
+  // allocates nothing on the host once its sizes have been seen
+  struct Group { int32_t mbase, nmem, pages, family, tile; bool split, reread; };
+  std::vector<Group> groups;
+  std::vector<int32_t> fam_of, fam_ids, by_fam, shared, own_pages, own_tokens, ns, item_family, order;
+  std::vector<AttnItem> sorted;
+};
+
 }  // namespace
 
 struct st_pool {
@@ -150,6 +171,9 @@ struct st_pool {
   std::vector<PendingTiming> pending;
   std::vector<cudaEvent_t> spare_events;
   std::string err;
+  // host scratch of st_decode_attn / st_decode_plan, reused call after call
+  DecodePlan plan;
+  std::vector<int> call_slots;
 };
 
 namespace {
@@ -698,94 +722,92 @@ ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok,
 
 namespace {
 
-// The decode work decomposition of one st_decode_attn call (host only; the
-// same plan st_decode_plan reports).  Branches are grouped by fork family and
+// Plans one st_decode_attn call.  Branches are grouped by fork family and
 // the full pages every member of a group holds (the longest common prefix of
 // their block tables) are read once for all of them; each branch's own pages
 // are read for it alone.  Runs of pages are sized to the SM count (about 64
 // waves of two CTAs per SM, at least 16 pages), the tile shape follows the
-// stacked rows (narrow up to 48, wide up to 128, balanced wide subgroups
-// beyond), and the items come out narrow first, longest first.
-struct DecodePlan {
-  std::vector<AttnItem> items;
-  std::vector<int32_t> members;   // the call's branch index of each item's members
-  std::vector<int32_t> n_splits;  // partials per branch
-  // algorithmic, whole launch: every KV page once per fork family and layer
-  // (shared pages once for the family, own pages once for their branch) and
-  // the queries
-  double bytes = 0, flops = 0;
-  double reread_bytes = 0;        // second and later reads of a split family's pages
-  double part_bytes = 0;          // the split-KV partials (written here, read by the combine)
-};
-
+// stacked rows (narrow up to 48, wide up to 128, paired up to 256, balanced
+// paired subgroups beyond), and the items come out narrow first, then wide,
+// then paired, longest first within each.
 void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   BlockPool& bp = *P->pool;
   const st_config& c = P->cfg;
   const int G = c.n_q_heads / c.n_kv_heads;
   const int n_br = (int)slots.size();
+  DecodePlan& d = *out;
   // ---- group by fork family, find the shared full pages --------------------
-  std::vector<int32_t> shared(n_br, 0);   // pages of branch i read through its group
-  struct Group { std::vector<int> members; int32_t pages; int32_t family; bool split, wide, reread; };
-  std::vector<Group> groups;
-  {
-    std::map<int32_t, std::vector<int>> fam;
-    std::vector<int32_t> order;
-    for (int i = 0; i < n_br; ++i) {
-      const int32_t f = bp.slot(slots[i]).family;
-      if (!fam.count(f)) order.push_back(f);
-      fam[f].push_back(i);
-    }
-    for (int32_t f : order) {
-      const std::vector<int>& mem = fam[f];
-      // one narrow tile (<= 48 stacked rows), else one wide tile (<= 128), else
-      // wide subgroups
-      const bool wide = (int)mem.size() * G > kMaxAttnRows;
-      const int per_group = std::max(1, (wide ? kMaxWideRows : kMaxAttnRows) / G);
-      // full pages held by every member of mem[b0, b1)
-      auto common_pages = [&](size_t b0, size_t b1) {
-        const SeqSlot& lead = bp.slot(slots[mem[b0]]);
-        int64_t min_len = lead.len;
-        int32_t pages = (int32_t)lead.table.size();
-        for (size_t x = b0 + 1; x < b1; ++x) {
-          const SeqSlot& ss = bp.slot(slots[mem[x]]);
-          pages = std::min(pages, lcp_pages(lead.table, ss.table));
-          min_len = std::min<int64_t>(min_len, ss.len);
-        }
-        return std::min<int32_t>(pages, (int32_t)(min_len / kPageTokens));
-      };
-      // A family larger than one tile is split into ceil(m / per_group)
-      // subgroups of near-equal size (7 at 6 per tile: 4 + 3), every one of
-      // them over the family's common pages, so that sibling items cover the
-      // same runs and can be scheduled together.
-      const size_t nm = mem.size(), n_sub = (nm + per_group - 1) / per_group;
-      const int32_t fam_pages = n_sub > 1 ? common_pages(0, nm) : 0;
-      for (size_t sg = 0; sg < n_sub; ++sg) {
-        const size_t b0 = sg * nm / n_sub, b1 = (sg + 1) * nm / n_sub;
-        if (n_sub == 1 && b1 - b0 < 2) continue;  // a lone sequence reads its pages as its own
-        const int32_t pages = n_sub > 1 ? fam_pages : common_pages(b0, b1);
-        if (pages < 1) continue;
-        Group g;
-        g.members.assign(mem.begin() + b0, mem.begin() + b1);
-        g.pages = pages;
-        g.family = f;
-        g.split = n_sub > 1;
-        g.wide = wide;
-        g.reread = sg > 0;  // the family's pages were counted with its first subgroup
-        for (int i : g.members) shared[i] = pages;
-        groups.push_back(std::move(g));
+  // by_fam: the call's branch indices ordered by family (families in order of
+  // first appearance, branches in call order within one)
+  d.fam_ids.clear();
+  d.fam_of.assign(n_br, 0);
+  for (int i = 0; i < n_br; ++i) {
+    const int32_t f = bp.slot(slots[i]).family;
+    int k = 0;
+    while (k < (int)d.fam_ids.size() && d.fam_ids[k] != f) ++k;
+    if (k == (int)d.fam_ids.size()) d.fam_ids.push_back(f);
+    d.fam_of[i] = k;
+  }
+  d.by_fam.clear();
+  for (int k = 0; k < (int)d.fam_ids.size(); ++k)
+    for (int i = 0; i < n_br; ++i)
+      if (d.fam_of[i] == k) d.by_fam.push_back(i);
+  d.shared.assign(n_br, 0);  // pages of branch i read through its group
+  d.groups.clear();
+  d.members.clear();
+  for (int k = 0, f0 = 0; k < (int)d.fam_ids.size(); ++k) {
+    int nm = 0;
+    while (f0 + nm < n_br && d.fam_of[d.by_fam[f0 + nm]] == k) ++nm;
+    const int32_t* mem = d.by_fam.data() + f0;
+    f0 += nm;
+    // one narrow tile (<= 48 stacked rows), else one wide tile (<= 128), else
+    // one paired tile (<= 256), else paired subgroups
+    const int rows = nm * G;
+    const int tile = rows <= kMaxAttnRows ? 0 : rows <= kMaxWideRows ? 1 : 2;
+    const int per_group = std::max(1, (tile == 0 ? kMaxAttnRows : tile == 1 ? kMaxWideRows : kMaxPairRows) / G);
+    // full pages held by every member of mem[b0, b1)
+    auto common_pages = [&](int b0, int b1) {
+      const SeqSlot& lead = bp.slot(slots[mem[b0]]);
+      int64_t min_len = lead.len;
+      int32_t pages = (int32_t)lead.table.size();
+      for (int x = b0 + 1; x < b1; ++x) {
+        const SeqSlot& ss = bp.slot(slots[mem[x]]);
+        pages = std::min(pages, lcp_pages(lead.table, ss.table));
+        min_len = std::min<int64_t>(min_len, ss.len);
+      }
+      return std::min<int32_t>(pages, (int32_t)(min_len / kPageTokens));
+    };
+    // A family larger than one tile is split into ceil(m / per_group)
+    // subgroups of near-equal size (40 at 32 per tile: 20 + 20), every one
+    // of them over the family's common pages, so that sibling items cover
+    // the same runs and can be scheduled together.
+    const int n_sub = (nm + per_group - 1) / per_group;
+    const int32_t fam_pages = n_sub > 1 ? common_pages(0, nm) : 0;
+    for (int sg = 0; sg < n_sub; ++sg) {
+      const int b0 = sg * nm / n_sub, b1 = (sg + 1) * nm / n_sub;
+      if (n_sub == 1 && b1 - b0 < 2) continue;  // a lone sequence reads its pages as its own
+      const int32_t pages = n_sub > 1 ? fam_pages : common_pages(b0, b1);
+      if (pages < 1) continue;
+      // the family's pages are counted (as algorithmic bytes) with its first subgroup
+      d.groups.push_back(DecodePlan::Group{(int32_t)d.members.size(), b1 - b0, pages, d.fam_ids[k], tile,
+                                           n_sub > 1, sg > 0});
+      for (int x = b0; x < b1; ++x) {
+        d.members.push_back(mem[x]);
+        d.shared[mem[x]] = pages;
       }
     }
   }
 
   // ---- chunking -------------------------------------------------------------
   int64_t total_pages = 0;
-  for (auto& g : groups) total_pages += g.pages;
-  std::vector<int32_t> own_pages(n_br), own_tokens(n_br);
+  for (const auto& g : d.groups) total_pages += g.pages;
+  d.own_pages.resize(n_br);
+  d.own_tokens.resize(n_br);
   for (int i = 0; i < n_br; ++i) {
     const SeqSlot& ss = bp.slot(slots[i]);
-    own_pages[i] = (int32_t)ss.table.size() - shared[i];
-    own_tokens[i] = (int32_t)(ss.len - (int64_t)shared[i] * kPageTokens);
-    total_pages += own_pages[i];
+    d.own_pages[i] = (int32_t)ss.table.size() - d.shared[i];
+    d.own_tokens[i] = (int32_t)(ss.len - (int64_t)d.shared[i] * kPageTokens);
+    total_pages += d.own_pages[i];
   }
   const int64_t units = total_pages * c.n_kv_heads * c.n_layers;
   // a metadata-only pool has no device: it plans for a GB300 (152 SMs, two decode CTAs each)
@@ -802,14 +824,14 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   // CTAs the runs of a given length make (the items below, times heads and layers)
   auto ctas_for = [&](int64_t ch) {
     int64_t n = 0;
-    std::vector<int32_t> ns(n_br, 0);
-    for (auto& g : groups) {
+    d.ns.assign(n_br, 0);
+    for (const auto& g : d.groups) {
       const int64_t k = std::min<int64_t>(max_prefix_chunks, (g.pages + ch - 1) / ch);
       n += k;
-      for (int i : g.members) ns[i] = (int32_t)k;
+      for (int x = 0; x < g.nmem; ++x) d.ns[d.members[g.mbase + x]] = (int32_t)k;
     }
     for (int i = 0; i < n_br; ++i)
-      if (own_pages[i] > 0) n += std::min<int64_t>(c.max_splits - ns[i], (own_pages[i] + ch - 1) / ch);
+      if (d.own_pages[i] > 0) n += std::min<int64_t>(c.max_splits - d.ns[i], (d.own_pages[i] + ch - 1) / ch);
     return n * c.n_kv_heads * c.n_layers;
   };
   // A small launch (a few waves) whose last wave is less than half full: longer
@@ -827,76 +849,87 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
     }
   }
 
-  std::vector<AttnItem> items;
-  std::vector<int32_t> item_family;  // fork family of a subgroup's item, for scheduling siblings together
-  std::vector<int32_t> members;
-  std::vector<int32_t> n_splits(n_br, 0);
+  std::vector<AttnItem>& items = d.items;
+  items.clear();
+  d.item_family.clear();  // fork family of a subgroup's item, for scheduling siblings together
+  d.n_splits.assign(n_br, 0);
   double bytes = 0, flops = 0, reread = 0;
   const double page_bytes = (double)kPageTokens * c.head_dim * 2 * 2;  // K+V, one head
-  for (auto& g : groups) {
+  for (const auto& g : d.groups) {
     const int32_t k = (int32_t)std::min<int64_t>(max_prefix_chunks, (g.pages + chunk - 1) / chunk);
-    const int32_t mbase = (int32_t)members.size();
-    for (int i : g.members) members.push_back(i);
+    const int32_t lead = d.members[g.mbase];
     for (int32_t cidx = 0; cidx < k; ++cidx) {
       int32_t b, n;
       split_even(g.pages, k, cidx, &b, &n);
-      items.push_back(AttnItem{slots[g.members[0]], b, n, n * kPageTokens, mbase, (int32_t)g.members.size(),
-                               cidx, (g.split ? kItemReread : 0) | (g.wide ? kItemWide : 0)});
-      item_family.push_back(g.family);
+      items.push_back(AttnItem{slots[lead], b, n, n * kPageTokens, g.mbase, g.nmem, cidx,
+                               (g.split ? kItemReread : 0) | (g.tile == 1 ? kItemWide : g.tile == 2 ? kItemPair : 0)});
+      d.item_family.push_back(g.family);
       (g.reread ? reread : bytes) += n * page_bytes;
-      flops += 4.0 * g.members.size() * G * n * kPageTokens * c.head_dim;
+      flops += 4.0 * g.nmem * G * n * kPageTokens * c.head_dim;
     }
-    for (int i : g.members) n_splits[i] = k;
+    for (int x = 0; x < g.nmem; ++x) d.n_splits[d.members[g.mbase + x]] = k;
   }
   for (int i = 0; i < n_br; ++i) {
-    if (own_pages[i] <= 0) continue;
-    const int32_t room = c.max_splits - n_splits[i];
-    const int32_t k = (int32_t)std::min<int64_t>(room, (own_pages[i] + chunk - 1) / chunk);
-    const int32_t mbase = (int32_t)members.size();
-    members.push_back(i);
+    if (d.own_pages[i] <= 0) continue;
+    const int32_t room = c.max_splits - d.n_splits[i];
+    const int32_t k = (int32_t)std::min<int64_t>(room, (d.own_pages[i] + chunk - 1) / chunk);
+    const int32_t mbase = (int32_t)d.members.size();
+    d.members.push_back(i);
     for (int32_t cidx = 0; cidx < k; ++cidx) {
       int32_t b, n;
-      split_even(own_pages[i], k, cidx, &b, &n);
-      const int32_t tok = std::min<int32_t>(n * kPageTokens, own_tokens[i] - b * kPageTokens);
-      items.push_back(AttnItem{slots[i], shared[i] + b, n, tok, mbase, 1, n_splits[i] + cidx, 0});
-      item_family.push_back(-1);
+      split_even(d.own_pages[i], k, cidx, &b, &n);
+      const int32_t tok = std::min<int32_t>(n * kPageTokens, d.own_tokens[i] - b * kPageTokens);
+      items.push_back(AttnItem{slots[i], d.shared[i] + b, n, tok, mbase, 1, d.n_splits[i] + cidx, 0});
+      d.item_family.push_back(-1);
       bytes += n * page_bytes;
       flops += 4.0 * G * tok * c.head_dim;
     }
-    n_splits[i] += k;
+    d.n_splits[i] += k;
   }
-  // narrow items, then wide ones (two launches); within each, longest runs
-  // first so the short ones fill the tail, and the items of a split group's
-  // subgroups over the same pages next to each other (same length, family and
-  // first page), so that the second read hits L2
+  // narrow items, then wide ones, then paired ones (up to three launches);
+  // within each, longest runs first so the short ones fill the tail, and the
+  // items of a split group's subgroups over the same pages next to each other
+  // (same length, family and first page), so that the second read hits L2.
+  // A stable order: an insertion sort for the usual few dozen items.
   {
-    std::vector<int> order(items.size());
-    for (size_t i = 0; i < order.size(); ++i) order[i] = (int)i;
     auto key = [&](int i) {
       const AttnItem& a = items[i];
       const bool rr = (a.flags & kItemReread) != 0;
-      return std::make_tuple((a.flags & kItemWide) ? 1 : 0, -a.n_pages, rr ? 0 : 1, rr ? item_family[i] : 0,
-                             rr ? a.page_begin : 0);
+      return std::make_tuple((a.flags & kItemPair) ? 2 : (a.flags & kItemWide) ? 1 : 0, -a.n_pages, rr ? 0 : 1,
+                             rr ? d.item_family[i] : 0, rr ? a.page_begin : 0);
     };
-    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return key(a) < key(b); });
-    std::vector<AttnItem> sorted(items.size());
-    for (size_t i = 0; i < order.size(); ++i) sorted[i] = items[order[i]];
-    items.swap(sorted);
+    const int n_items = (int)items.size();
+    d.order.resize(n_items);
+    for (int i = 0; i < n_items; ++i) d.order[i] = i;
+    auto less = [&](int a, int b) { return key(a) < key(b); };
+    if (n_items <= 128) {
+      for (int i = 1; i < n_items; ++i) {
+        const int v = d.order[i];
+        int j = i;
+        while (j > 0 && less(v, d.order[j - 1])) {
+          d.order[j] = d.order[j - 1];
+          --j;
+        }
+        d.order[j] = v;
+      }
+    } else {
+      std::stable_sort(d.order.begin(), d.order.end(), less);
+    }
+    d.sorted.resize(n_items);
+    for (int i = 0; i < n_items; ++i) d.sorted[i] = items[d.order[i]];
+    items.swap(d.sorted);
   }
   bytes *= (double)c.n_kv_heads * c.n_layers;
   reread *= (double)c.n_kv_heads * c.n_layers;
   flops *= (double)c.n_kv_heads * c.n_layers;
   const double q_bytes = (double)c.n_layers * n_br * c.n_q_heads * c.head_dim * 2;
   double part_rows = 0;
-  for (auto& it : items) part_rows += (double)it.n_members * G;
+  for (const auto& it : items) part_rows += (double)it.n_members * G;
   part_rows *= (double)c.n_kv_heads * c.n_layers;
-  out->items = std::move(items);
-  out->members = std::move(members);
-  out->n_splits = std::move(n_splits);
-  out->bytes = bytes + q_bytes;
-  out->flops = flops;
-  out->reread_bytes = reread;
-  out->part_bytes = part_rows * (c.head_dim + 1) * 4;
+  d.bytes = bytes + q_bytes;
+  d.flops = flops;
+  d.reread_bytes = reread;
+  d.part_bytes = part_rows * (c.head_dim + 1) * 4;
 }
 
 // The call's branches as pool slots: live, non-empty, each listed once.
@@ -924,7 +957,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
   if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
     return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
-  std::vector<int> slots;
+  std::vector<int>& slots = P->call_slots;
   st_status vs = decode_slots(P, br, n_br, &slots);
   if (vs != ST_OK) return vs;
   const st_config& c = P->cfg;
@@ -932,7 +965,7 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   DeviceGuard guard(P->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
 
-  DecodePlan dp;
+  DecodePlan& dp = P->plan;
   plan_decode(P, slots, &dp);
   const std::vector<AttnItem>& items = dp.items;
   const std::vector<int32_t>& members = dp.members;
@@ -996,16 +1029,21 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   // few: the next step reads the same pages, so they stay in L2
   ap.keep_l2 = bytes < 0.5 * (double)P->l2_bytes ? 1 : 0;
   const int n_items = (int)items.size();
-  int n_narrow = 0;
-  while (n_narrow < n_items && !(items[n_narrow].flags & kItemWide)) ++n_narrow;
+  int n_narrow = 0, n_wide = 0;
+  while (n_narrow < n_items && !(items[n_narrow].flags & (kItemWide | kItemPair))) ++n_narrow;
+  while (n_narrow + n_wide < n_items && (items[n_narrow + n_wide].flags & kItemWide)) ++n_wide;
+  const int n_pair = n_items - n_narrow - n_wide;
   st = run_kernel(P, kKDecode, bytes, flops, s, [&] {
     const InlineDecodePlan* ip = inline_plan ? &inl : nullptr;
     cudaError_t e = launch_decode_tc(P->kmap, P->vmap, ap, ip, n_narrow, c.head_dim, false, s);
-    if (e != cudaSuccess || n_narrow == n_items) return e;
+    if (e != cudaSuccess) return e;
     AttnParams aw = ap;
     aw.item_base = n_narrow;
-    return launch_decode_tc(P->kmap, P->vmap, aw, ip, n_items - n_narrow, c.head_dim, true, s);
-  }, (n_narrow > 0 ? 1 : 0) + (n_items > n_narrow ? 1 : 0), dp.reread_bytes + part_bytes);
+    e = launch_decode_tc(P->kmap, P->vmap, aw, ip, n_wide, c.head_dim, true, s);
+    if (e != cudaSuccess) return e;
+    aw.item_base = n_narrow + n_wide;
+    return launch_decode_pair(P->kmap, P->vmap, aw, ip, n_pair, c.head_dim, s);
+  }, (n_narrow > 0 ? 1 : 0) + (n_wide > 0 ? 1 : 0) + (n_pair > 0 ? 1 : 0), dp.reread_bytes + part_bytes);
   if (st != ST_OK) {
     if (ps >= 0) retire_plan(P, ps, s);  // its copy may still be in flight
     return st;
@@ -1036,10 +1074,10 @@ ST_API st_status st_decode_plan(st_pool* P, const st_seq* br, int n_br, int32_t*
                                 int32_t* members, int member_cap, int32_t* n_splits, int* n_items,
                                 int* n_members) {
   if (!P) return ST_ERR_INVALID;
-  std::vector<int> slots;
+  std::vector<int>& slots = P->call_slots;
   st_status vs = decode_slots(P, br, n_br, &slots);
   if (vs != ST_OK) return vs;
-  DecodePlan dp;
+  DecodePlan& dp = P->plan;
   plan_decode(P, slots, &dp);
   if (n_items) *n_items = (int)dp.items.size();
   if (n_members) *n_members = (int)dp.members.size();

@@ -9,8 +9,8 @@ import pytest
 import paper_2608_13667_gb300 as stpkg
 
 PAGE = 16
-NARROW_ROWS, WIDE_ROWS = 48, 128
-WIDE, REREAD = 2, 1
+NARROW_ROWS, WIDE_ROWS, PAIR_ROWS = 48, 128, 256
+WIDE, REREAD, PAIR = 2, 1, 4
 
 
 def _pool(G, Hkv, max_splits, n_blocks=1 << 15):
@@ -25,17 +25,18 @@ def check_plan(P, br, G, max_splits):
     covered = [dict() for _ in range(n)]   # logical page -> physical id, per branch
     tokens = [0] * n
     splits = [[] for _ in range(n)]
-    seen_wide = False
+    last_tile = 0
     for it in items:
         mem = members[it["member_base"]:it["member_base"] + it["n_members"]]
         own = tables[it["owner"]]
         p0, np_ = it["page_begin"], it["n_pages"]
         assert np_ >= 1 and it["n_tokens"] >= 1
-        wide = bool(it["flags"] & WIDE)
-        assert len(mem) * G <= (WIDE_ROWS if wide else NARROW_ROWS)
-        assert not (it["flags"] & REREAD) or wide
-        assert not (seen_wide and not wide), "narrow items come before wide ones"
-        seen_wide |= wide
+        tile = 2 if it["flags"] & PAIR else 1 if it["flags"] & WIDE else 0
+        assert not (it["flags"] & PAIR and it["flags"] & WIDE)
+        assert len(mem) * G <= (NARROW_ROWS, WIDE_ROWS, PAIR_ROWS)[tile]
+        assert not (it["flags"] & REREAD) or tile == 2, "only families beyond one paired tile are split"
+        assert tile >= last_tile, "narrow items first, then wide, then paired"
+        last_tile = tile
         if len(mem) > 1:
             assert it["n_tokens"] == np_ * PAGE   # a shared run holds full pages only
         else:
@@ -109,11 +110,12 @@ def test_shared_prefix_is_read_once_per_group(stlib):
     assert all(it["n_members"] == 5 and not it["flags"] & WIDE for it in shared)
 
 
-@pytest.mark.parametrize("n_br,G,tiles", [(6, 8, 1), (16, 8, 1), (17, 8, 2), (40, 4, 2), (9, 16, 2)])
+@pytest.mark.parametrize("n_br,G,tiles", [(6, 8, 1), (16, 8, 1), (17, 8, 1), (40, 4, 1), (9, 16, 1), (32, 8, 1),
+                                         (33, 8, 2), (48, 8, 2), (6, 48, 2), (48, 16, 3)])
 def test_tile_choice_follows_the_stacked_rows(stlib, n_br, G, tiles):
-    """Up to 48 stacked rows: narrow; up to 128: one wide tile; beyond:
-    balanced wide subgroups, each over the family's common pages, flagged so
-    the sibling's read of a page comes from L2."""
+    """Up to 48 stacked rows: narrow; up to 128: one wide tile; up to 256: one
+    paired tile; beyond: balanced paired subgroups, each over the family's
+    common pages, flagged so the sibling's read of a page comes from L2."""
     P = _pool(G, 1, 32)
     m = P.seq_create()
     P.append_kv([m], 4096, None)
@@ -125,7 +127,8 @@ def test_tile_choice_follows_the_stacked_rows(stlib, n_br, G, tiles):
     groups = {it["member_base"] for it in shared}
     assert len(groups) == tiles
     rows = n_br * G
-    assert all(bool(it["flags"] & WIDE) == (rows > NARROW_ROWS) for it in shared)
+    assert all(bool(it["flags"] & WIDE) == (NARROW_ROWS < rows <= WIDE_ROWS) for it in shared)
+    assert all(bool(it["flags"] & PAIR) == (rows > WIDE_ROWS) for it in shared)
     assert all(bool(it["flags"] & REREAD) == (tiles > 1) for it in shared)
     if tiles > 1:
         sizes = sorted(it["n_members"] for it in shared if it["split"] == 0)

@@ -256,6 +256,33 @@ def test_shapes(stlib, D, Hq, Hkv, n_aux, P, suffix):
         compare(o[layer], lse[layer], o_ref, l_ref, f"layer {layer}")
 
 
+@pytest.mark.parametrize("D,Hq,Hkv,n_br,P", [
+    (128, 64, 8, 17, 3000),    # G = 8, 136 rows: one paired tile, its second tile 8 rows
+    (128, 128, 8, 16, 2000),   # G = 16, 256 rows: a full paired tile
+    (64, 48, 16, 43, 1500),    # G = 3, 129 rows
+    (128, 64, 8, 40, 5000),    # 320 rows: two paired subgroups of 160
+    (64, 32, 2, 20, 777),      # G = 16, D 64, 320 rows
+])
+def test_large_fork_groups(stlib, D, Hq, Hkv, n_br, P):
+    """Fork groups beyond 128 stacked rows: one paired tile (two M = 128 tiles
+    of one CTA over every stage) up to 256, balanced paired subgroups beyond,
+    each branch with a suffix of its own; every layer against the oracle."""
+    w = _small(D, Hq, Hkv, n_blocks=4096, L=2, seed=13)
+    run = Run(w, max_seqs=64, max_decode_branches=48, max_splits=8)
+    m = run.create()
+    run.append([m], P, ("prefix",))
+    br = [m] + run.fork(m, n_br - 1)
+    for b, rid in enumerate(br):
+        if b % 3 and (7 * b) % 41:
+            run.append([rid], (7 * b) % 41, ("suffix", b))
+    q, o, lse = run.decode(br, ("q",))
+    run.pool.sync()
+    run.check_tables()
+    for layer in range(w.n_layers):
+        o_ref, l_ref = run.oracle_decode(br, q, layer)
+        compare(o[layer], lse[layer], o_ref, l_ref, f"{n_br} branches, layer {layer}")
+
+
 def test_many_splits_on_a_long_singleton(stlib):
     w = _small(128, 32, 8, n_blocks=4096, L=1)
     run = Run(w, max_seqs=4, max_decode_branches=4, max_splits=32)
