@@ -361,6 +361,8 @@ def run_ours(args, rank, ws, local):
                     "copies": "pinned host buffers, H2D and D2H on their own streams, double-buffered, "
                               "overlapping the neighbouring steps' compute"},
         }
+        if step_bytes < 0.5 * L2_BYTES:
+            res["latency"] = _c_abi_latency(pool, br, step_k, step_v, step_q, o, lse, args.steps, dev)
     pool.close()
     if rank == 0:
         # the tensor-bound half of the path: the merge prefill, timed alone on a
@@ -376,6 +378,44 @@ def run_ours(args, rank, ws, local):
                          "flops": "algorithmic: 4 D x causal keys x q heads x layers; P V runs for both bf16 "
                                   "terms of P, so the tensor cores execute 1.5x this"}}
     return res
+
+
+def _c_abi_latency(pool, br, step_k, step_v, step_q, o, lse, n, dev):
+    """A step of the latency case (a working set that stays in L2) timed through
+    the C ABI alone: st_append_kv and st_decode_attn called with arguments
+    marshalled once, no per-kernel events.  Returns microseconds per step."""
+    import ctypes
+    import torch
+    import paper_2608_13667_gb300 as st
+    L = st.lib()
+    h = pool._h
+    arr, n_br = st._seq_array(br)
+    sp = pool._stream(None)
+    vp = lambda t: ctypes.c_void_p(t.data_ptr())
+    ks, vs, qs = [vp(t) for t in step_k], [vp(t) for t in step_v], [vp(t) for t in step_q]
+    op, lp = vp(o), vp(lse)
+    m = len(ks)
+
+    def run(count):
+        for s in range(count):
+            if L.st_append_kv(h, arr, n_br, 1, ks[s % m], vs[s % m], sp) or \
+                    L.st_decode_attn(h, arr, n_br, qs[s % m], op, lp, sp):
+                raise RuntimeError(L.st_last_error(h).decode())
+
+    run(5)
+    stream = torch.cuda.current_stream(dev)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.perf_counter()
+    e0.record(stream)
+    run(n)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    host_s = time.perf_counter() - t0
+    pool.sync()
+    return {"us_per_step": e0.elapsed_time(e1) * 1e3 / n, "host_us_per_step": host_s * 1e6 / n, "steps": n,
+            "how": "append + decode of every branch per step, st_append_kv and st_decode_attn called from a "
+                   "ctypes loop with arguments marshalled once, no per-kernel events; the step's pages stay in L2"}
 
 
 # --------------------------------------------------------------------------- profiling case

@@ -16,8 +16,7 @@ namespace {
 // One warp per (layer, branch, query head): lse = log sum_i exp(lse_i),
 // O = sum_i exp(lse_i - lse) O_i over the branch's partials.
 template <int D>
-__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
-                                                      const __grid_constant__ InlineDecodePlan inl) {
+__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p, const __grid_constant__ InlineSplits inl) {
   griddep_wait();
   griddep_launch_dependents();
   const int32_t* n_splits = p.n_splits ? p.n_splits : inl.n_splits;
@@ -90,9 +89,9 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p,
 
 }  // namespace
 
-cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, int D, cudaStream_t s) {
-  static const InlineDecodePlan kNone{};
-  const InlineDecodePlan& ip = inl ? *inl : kNone;
+cudaError_t launch_combine(const CombineParams& p, const InlineSplits* inl, int D, cudaStream_t s) {
+  static const InlineSplits kNone{};
+  const InlineSplits& ip = inl ? *inl : kNone;
   const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
   if (total == 0) return cudaSuccess;
   const int grid = (int)((total + 3) / 4);

@@ -125,6 +125,10 @@ struct InlineDecodePlan {
   int32_t members[kInlineMembers];
   int32_t n_splits[kInlineBranches];
 };
+// the part of a small plan the combine reads (a smaller parameter block to launch)
+struct InlineSplits {
+  int32_t n_splits[kInlineBranches];
+};
 constexpr int kInlineAppendBranches = 32;
 constexpr int kInlineCows = 32;
 struct InlineAppendPlan {
@@ -167,7 +171,7 @@ cudaError_t launch_chained(void (*kernel)(KArgs...), dim3 grid, dim3 block, size
 cudaError_t launch_table_update(int32_t* table, const TableRun* runs, const int32_t* values,
                                 int n_runs, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, const InlineAppendPlan* inl, int D, cudaStream_t s);
-cudaError_t launch_combine(const CombineParams& p, const InlineDecodePlan* inl, int D, cudaStream_t s);
+cudaError_t launch_combine(const CombineParams& p, const InlineSplits* inl, int D, cudaStream_t s);
 // Decode partials on tcgen05 (one CTA per item x KV head x layer; items from
 // p.item_base on; wide: the M = 128 tile, for items flagged kItemWide).
 cudaError_t launch_decode_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p,

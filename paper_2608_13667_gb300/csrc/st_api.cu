@@ -171,9 +171,12 @@ struct st_pool {
   std::vector<PendingTiming> pending;
   std::vector<cudaEvent_t> spare_events;
   std::string err;
-  // host scratch of st_decode_attn / st_decode_plan, reused call after call
+  // host scratch of the calls, reused call after call
   DecodePlan plan;
   std::vector<int> call_slots;
+  std::vector<int32_t> call_counts;
+  std::vector<AppendBranch> app_branches;
+  std::vector<CowEvent> app_cows;
 };
 
 namespace {
@@ -417,13 +420,15 @@ st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, in
   }
 
   // ---- from here on the host tables change ----------------------------------
-  std::vector<AppendBranch> brs(n_br);
+  std::vector<AppendBranch>& brs = P->app_branches;
+  brs.resize(n_br);
   int32_t row0 = 0;
   for (int i = 0; i < n_br; ++i) {
     brs[i] = AppendBranch{slots[i], (int32_t)bp.slot(slots[i]).len, row0, counts[i]};
     row0 += counts[i];
   }
-  std::vector<CowEvent> cows;
+  std::vector<CowEvent>& cows = P->app_cows;
+  cows.clear();
   if (uniform) {
     bp.append(slots, n_br, n_br ? counts[0] : 0, &cows);
   } else {
@@ -489,8 +494,8 @@ st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, in
 
 st_status do_append(st_pool* P, const int* slots, int n_br, int n_tok, const void* k, const void* v,
                     cudaStream_t s) {
-  std::vector<int32_t> counts(n_br, n_tok);
-  return do_append_rows(P, slots, counts.data(), n_br, k, v, s);
+  P->call_counts.assign(n_br, n_tok);
+  return do_append_rows(P, slots, P->call_counts.data(), n_br, k, v, s);
 }
 
 // Longest common prefix (in pages) of two block tables.
@@ -704,7 +709,8 @@ ST_API st_status st_append_kv(st_pool* P, const st_seq* br, int n_br, int n_tok,
   if (!P) return ST_ERR_INVALID;
   if (st_status b_ = refuse_if_broken(P)) return b_;
   if (n_br < 0 || n_tok < 0 || (n_br > 0 && !br)) return fail(P, ST_ERR_INVALID, "bad n_br/n_tok");
-  std::vector<int> slots(n_br);
+  std::vector<int>& slots = P->call_slots;
+  slots.resize(n_br);
   for (int i = 0; i < n_br; ++i) {
     if (!decode_handle(P, br[i], &slots[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
     for (int j = 0; j < i; ++j)
@@ -1061,8 +1067,10 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   cp.max_splits = c.max_splits;
   // algorithmic: O and LSE written once; the partials it reads are the split's own traffic
   const double cbytes = (double)c.n_layers * n_br * c.n_q_heads * (c.head_dim + 1) * 4;
+  InlineSplits isp;
+  if (inline_plan) std::memcpy(isp.n_splits, n_splits.data(), n_br * sizeof(int32_t));
   st = run_kernel(P, kKCombine, cbytes, 0, s,
-                  [&] { return launch_combine(cp, inline_plan ? &inl : nullptr, c.head_dim, s); }, 1, part_bytes);
+                  [&] { return launch_combine(cp, inline_plan ? &isp : nullptr, c.head_dim, s); }, 1, part_bytes);
   if (st != ST_OK) {
     if (ps >= 0) retire_plan(P, ps, s);  // its copy may still be in flight
     return st;
