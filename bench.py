@@ -382,8 +382,10 @@ def run_ours(args, rank, ws, local):
 
 def _c_abi_latency(pool, br, step_k, step_v, step_q, o, lse, n, dev):
     """A step of the latency case (a working set that stays in L2) timed through
-    the C ABI alone: st_append_kv and st_decode_attn called with arguments
-    marshalled once, no per-kernel events.  Returns microseconds per step."""
+    the C ABI alone, with arguments marshalled once and no per-kernel events:
+    st_decode_step (one row appended per branch and the decode, the row
+    written by the decode kernel), and st_append_kv then st_decode_attn.
+    Returns microseconds per step for both."""
     import ctypes
     import torch
     import paper_2608_13667_gb300 as st
@@ -396,26 +398,34 @@ def _c_abi_latency(pool, br, step_k, step_v, step_q, o, lse, n, dev):
     op, lp = vp(o), vp(lse)
     m = len(ks)
 
-    def run(count):
-        for s in range(count):
-            if L.st_append_kv(h, arr, n_br, 1, ks[s % m], vs[s % m], sp) or \
-                    L.st_decode_attn(h, arr, n_br, qs[s % m], op, lp, sp):
-                raise RuntimeError(L.st_last_error(h).decode())
+    def fused(s):
+        return L.st_decode_step(h, arr, n_br, ks[s % m], vs[s % m], qs[s % m], op, lp, sp)
 
-    run(5)
+    def separate(s):
+        return L.st_append_kv(h, arr, n_br, 1, ks[s % m], vs[s % m], sp) or \
+            L.st_decode_attn(h, arr, n_br, qs[s % m], op, lp, sp)
+
     stream = torch.cuda.current_stream(dev)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t0 = time.perf_counter()
-    e0.record(stream)
-    run(n)
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    host_s = time.perf_counter() - t0
+    out = {}
+    for name, call in (("st_decode_step", fused), ("st_append_kv + st_decode_attn", separate)):
+        for s in range(5):
+            if call(s):
+                raise RuntimeError(L.st_last_error(h).decode())
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        e0.record(stream)
+        for s in range(n):
+            if call(s):
+                raise RuntimeError(L.st_last_error(h).decode())
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        out[name] = {"us_per_step": e0.elapsed_time(e1) * 1e3 / n,
+                     "host_us_per_step": (time.perf_counter() - t0) * 1e6 / n}
     pool.sync()
-    return {"us_per_step": e0.elapsed_time(e1) * 1e3 / n, "host_us_per_step": host_s * 1e6 / n, "steps": n,
-            "how": "append + decode of every branch per step, st_append_kv and st_decode_attn called from a "
-                   "ctypes loop with arguments marshalled once, no per-kernel events; the step's pages stay in L2"}
+    return {"us_per_step": out["st_decode_step"]["us_per_step"], "steps": n, "calls": out,
+            "how": "one row appended to every branch and the decode, per step, called from a ctypes loop with "
+                   "arguments marshalled once and no per-kernel events; the step's pages stay in L2"}
 
 
 # --------------------------------------------------------------------------- profiling case

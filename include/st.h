@@ -164,6 +164,21 @@ ST_API st_status st_append_kv(st_pool* pool, const st_seq* br, int n_br, int n_t
 ST_API st_status st_decode_attn(st_pool* pool, const st_seq* br, int n_br, const void* q, float* o,
                                 float* lse, void* stream);
 
+/* One step of the decode loop (Section 3.1: each branch generates its own
+ * tokens): append one KV row to each branch, then decode one query per
+ * branch -- the same result, tables and page allocation as st_append_kv with
+ * n_tok = 1 followed by st_decode_attn on the same branches, in fewer
+ * launches: the decode kernel that reads a branch's last page writes the new
+ * row into it first.  (When a branch's last page is shared and partly filled,
+ * the step copies it with a separate append launch first.)
+ * k, v: device bf16 [n_layers][n_br][n_kv_heads][head_dim], the new rows;
+ * q, o, lse: as st_decode_attn.  Branches may be empty before the call.
+ * Failures before the append change nothing; a failure after it (a CUDA
+ * error, or a plan too large for one staging slot) leaves the pool unusable,
+ * as for the other appending calls. */
+ST_API st_status st_decode_step(st_pool* pool, const st_seq* br, int n_br, const void* k, const void* v,
+                                const void* q, float* o, float* lse, void* stream);
+
 /* The work decomposition st_decode_attn would use for these branches, without
  * launching anything (host only; also on a metadata-only pool, which plans for
  * 152 SMs with two decode CTAs each).  One item is a run of pages of one

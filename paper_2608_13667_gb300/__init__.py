@@ -81,6 +81,7 @@ def lib():
         "st_append_kv": (I, [P, i64p, I, I, VP, VP, VP]),
         "st_decode_attn": (I, [P, i64p, I, VP, VP, VP, VP]),
         "st_decode_plan": (I, [P, i64p, I, i32p, I, i32p, I, i32p, ctypes.POINTER(I), ctypes.POINTER(I)]),
+        "st_decode_step": (I, [P, i64p, I, VP, VP, VP, VP, VP, VP]),
         "st_merge": (I, [P, I64, I, VP, VP, VP, VP, VP, VP]),
         "st_prefill_batch": (I, [P, i64p, I, i32p, VP, VP, VP, VP, VP, VP]),
         "st_release": (I, [P, I64]),
@@ -257,6 +258,26 @@ class Pool:
         self._check(lib().st_decode_attn(self._h, arr, n, qp, op, lp, self._stream(stream)), "st_decode_attn")
         return o, lse
 
+    def decode_step(self, branches, k, v, q, o=None, lse=None, stream=None):
+        """One decode step: append one row per branch (k, v: bf16 [L][n_br][Hkv][D])
+        and decode q (bf16 [L][n_br][Hq][D]) -> (o, lse), as st_append_kv then
+        st_decode_attn."""
+        import torch
+        arr, n = self._seqs(branches)
+        c = self.cfg
+        kp = self._dev(k, torch.bfloat16, (c.n_layers, n, c.n_kv_heads, c.head_dim), "k")
+        vp = self._dev(v, torch.bfloat16, (c.n_layers, n, c.n_kv_heads, c.head_dim), "v")
+        qp = self._dev(q, torch.bfloat16, (c.n_layers, n, c.n_q_heads, c.head_dim), "q")
+        if o is None:
+            o = torch.empty((c.n_layers, n, c.n_q_heads, c.head_dim), dtype=torch.float32, device=self.device)
+        if lse is None:
+            lse = torch.empty((c.n_layers, n, c.n_q_heads), dtype=torch.float32, device=self.device)
+        op = self._dev(o, torch.float32, (c.n_layers, n, c.n_q_heads, c.head_dim), "o")
+        lp = self._dev(lse, torch.float32, (c.n_layers, n, c.n_q_heads), "lse")
+        self._check(lib().st_decode_step(self._h, arr, n, kp, vp, qp, op, lp, self._stream(stream)),
+                    "st_decode_step")
+        return o, lse
+
     def decode_plan(self, branches):
         """The work decomposition st_decode_attn uses for these branches (host
         only, also on a metadata-only pool): (items, members, n_splits), items a
@@ -391,6 +412,10 @@ def st_append_kv(pool, branches, k, v, stream=None):
 
 def st_decode_attn(pool, branches, q, o=None, lse=None, stream=None):
     return pool.decode_attn(branches, q, o, lse, stream)
+
+
+def st_decode_step(pool, branches, k, v, q, o=None, lse=None, stream=None):
+    return pool.decode_step(branches, k, v, q, o, lse, stream)
 
 
 def st_merge(pool, main, q, k, v, o=None, lse=None, stream=None):

@@ -39,6 +39,12 @@
 //               Narrow: one ring, a stage's K and V slots freed together after
 //               its P V.  Wide: K and V have their own barriers; a K slot is
 //               freed by the commit after S_j, a V slot after P_j V_j.
+//               A decode step (st_decode_step): the narrow item that holds a
+//               branch's last page first stores the step's new K and V row of
+//               its (layer, KV head) into that page, then a proxy fence makes
+//               the store visible to the page's TMA copies.  Only that CTA
+//               reads the page (a branch's last page is its own), so no
+//               separate append launch is needed.
 //   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M, N=64 keys)
 //               and O += P V (M, N=D) and commits them to mbarriers.  S is
 //               double-buffered in TMEM: S_{j+1} is issued before P_j V_j when
@@ -275,6 +281,29 @@ __global__ void __launch_bounds__(kThreads, 2)
           nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
         }
         const int np = min(C::kPagesPerStage, n_pages - page0);
+        if ((item.flags & kItemAppend) && jk == n_tiles - 1) {
+          // a decode step: this run's last key is the row the step appends.
+          // The warp writes this (layer, KV head)'s K and V of it into the
+          // pool (16 bytes per lane), then makes the writes visible to the
+          // copies below, which load that page.
+          const int last = n_valid_keys - 1 - page0 * kPageTokens;  // key within the stage
+          int blk = __shfl_sync(0xffffffffu, cur, (page0 - base_id + last / kPageTokens) & 31);
+          constexpr int kChunks = D / 8;
+          if (lane < 2 * kChunks) {
+            if ((uint64_t)blk >= (uint64_t)p.n_blocks) {
+              atomicCAS(p.status, 0, kDevBadIndex);
+            } else {
+              const bool is_v = lane >= kChunks;
+              const int c = lane % kChunks;
+              const int64_t src = (((int64_t)layer * p.n_rows_q + members[item.member_base]) * p.Hkv + kvh) * D + c * 8;
+              const int64_t dst =
+                  ((((int64_t)layer * p.n_blocks + blk) * p.Hkv + kvh) * kPageTokens + last % kPageTokens) * D + c * 8;
+              *reinterpret_cast<uint4*>((is_v ? p.v_pool : p.k_pool) + dst) =
+                  *reinterpret_cast<const uint4*>((is_v ? p.app_v : p.app_k) + src);
+              fence_proxy_async_global();
+            }
+          }
+        }
         if (lane == 0) mbar_arrive_expect_tx(&full[s], 2 * np * page_bytes);
         __syncwarp();
         // one copy per lane (lane = 2 D/64 q + (V ? D/64 : 0) + h): a single

@@ -13,34 +13,26 @@ namespace st {
 
 namespace {
 
-// One warp per (layer, branch, query head): lse = log sum_i exp(lse_i),
-// O = sum_i exp(lse_i - lse) O_i over the branch's partials.
+// One row (one layer, branch and query head) for one warp: lse = log sum_i
+// exp(lse_i), O = sum_i exp(lse_i - lse) O_i over the row's ns partials
+// (ns <= 32).
 template <int D>
-__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p, const __grid_constant__ InlineSplits inl) {
-  griddep_wait();
-  griddep_launch_dependents();
-  const int32_t* n_splits = p.n_splits ? p.n_splits : inl.n_splits;
-  const int lane = threadIdx.x & 31;
-  const int64_t idx = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
-  const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
-  if (idx >= total) return;
-  const int b = (int)((idx / p.Hq) % p.n_br);
-  const int ns = n_splits[b];
+__device__ __forceinline__ void combine_row(const float* lse_i, const float* part_o, int ns, float* o_out,
+                                            float* lse_out, int lane) {
   constexpr int kPer = D / 32;
   constexpr int kBatch = 16;  // partials whose loads are in flight together
-  const float* lse_i = p.part_lse + idx * p.max_splits;
-  const float* po = p.part_o + idx * p.max_splits * D + lane * kPer;
-  // this lane's column slice of partial i (zero past the branch's partials)
+  const float* po = part_o + lane * kPer;
+  // this lane's column slice of partial i (zero past the row's partials)
   auto load = [&](int i, float* x) {
     if (i < ns) {
       if constexpr (kPer == 4) {
-        const float4 v = *reinterpret_cast<const float4*>(po + (int64_t)i * D);
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(po + (int64_t)i * D));
         x[0] = v.x;
         x[1] = v.y;
         x[2] = v.z;
         x[3] = v.w;
       } else {
-        const float2 v = *reinterpret_cast<const float2*>(po + (int64_t)i * D);
+        const float2 v = __ldcg(reinterpret_cast<const float2*>(po + (int64_t)i * D));
         x[0] = v.x;
         x[1] = v.y;
       }
@@ -51,17 +43,17 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p, con
   };
   // the first batch of partials is loaded together with the lse values: the
   // loads do not depend on the weights
-  const float li = lane < ns ? lse_i[lane] : -INFINITY;
+  const float li = lane < ns ? __ldcg(lse_i + lane) : -INFINITY;
   float x[kBatch][kPer];
 #pragma unroll
   for (int u = 0; u < kBatch; ++u) load(u, x[u]);
   float mx = li;
 #pragma unroll
-  for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  for (int off = 16; off; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   const float w = lane < ns ? expf(li - mx) : 0.f;
   float sum = w;
 #pragma unroll
-  for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  for (int off = 16; off; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
   const float lse = mx + logf(sum);
   const float inv_sum = 1.f / sum;
   float out[kPer];
@@ -79,12 +71,28 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineParams p, con
       for (int e = 0; e < kPer; ++e) out[e] += wv * x[u][e];
     }
   }
-  float* dst = p.o + idx * D + lane * kPer;
-  if (kPer == 4)
+  float* dst = o_out + lane * kPer;
+  if constexpr (kPer == 4)
     *reinterpret_cast<float4*>(dst) = make_float4(out[0], out[1], out[2], out[3]);
   else
     *reinterpret_cast<float2*>(dst) = make_float2(out[0], out[1]);
-  if (lane == 0) p.lse[idx] = lse;
+  if (lane == 0) *lse_out = lse;
+}
+
+
+// One warp per (layer, branch, query head).
+template <int D>
+__global__ void __launch_bounds__(128) combine_kernel(const CombineParams p, const __grid_constant__ InlineSplits inl) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int32_t* n_splits = p.n_splits ? p.n_splits : inl.n_splits;
+  const int lane = threadIdx.x & 31;
+  const int64_t idx = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int64_t total = (int64_t)p.L * p.n_br * p.Hq;
+  if (idx >= total) return;
+  const int b = (int)((idx / p.Hq) % p.n_br);
+  combine_row<D>(p.part_lse + idx * p.max_splits, p.part_o + idx * p.max_splits * D, n_splits[b], p.o + idx * D,
+                 p.lse + idx, lane);
 }
 
 }  // namespace

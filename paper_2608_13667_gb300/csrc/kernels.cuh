@@ -74,6 +74,9 @@ constexpr int32_t kItemWide = 2;
 // more than 128 stacked rows: two M = 128 tiles of one CTA sharing every K/V
 // stage (the merge's paired tile, merge_tc.cu)
 constexpr int32_t kItemPair = 4;
+// a decode step's own item whose last key is the row the step appends: its
+// loader writes that row into the pool before loading the page (st_decode_step)
+constexpr int32_t kItemAppend = 8;
 
 // One CTA of a batched merge / prefill: rows [row_base, row_base + 256) of
 // one sequence's stacked (new row, head) rows.
@@ -103,6 +106,12 @@ struct AttnParams {
   int32_t item_base;       // decode: CTA x reads item item_base + x
   int32_t keep_l2;         // decode: the launch's pages fit in L2; load them evict-normal so they stay
   const MergeItem* mitems; // batched merge: CTA x takes mitems[x] (slot, L0, T above unused)
+  // decode step (items flagged kItemAppend): the rows the step appends,
+  // [L][n_br][Hkv][D], and the pools they go to
+  const __nv_bfloat16* app_k;
+  const __nv_bfloat16* app_v;
+  __nv_bfloat16* k_pool;
+  __nv_bfloat16* v_pool;
 };
 
 struct CombineParams {

@@ -386,8 +386,12 @@ bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 // counts][Hkv][D].  All or nothing: capacity, the plan's size and its staging
 // slot are settled before any table changes; a CUDA failure after that
 // leaves the pool unusable (every later call returns ST_ERR_STATE).
+// With `deferred` non-null (a decode step of one row per branch), the rows
+// are left to the decode kernels when the append needs no copy-on-write:
+// *deferred is then set and no append kernel is launched.
 st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, int n_br, const void* k,
-                         const void* v, cudaStream_t s) {
+                         const void* v, cudaStream_t s, bool* deferred = nullptr) {
+  if (deferred) *deferred = false;
   BlockPool& bp = *P->pool;
   int64_t need = 0, n_rows = 0;
   int cow_bound = 0;  // branches whose append may start with a copy-on-write
@@ -438,6 +442,11 @@ st_status do_append_rows(st_pool* P, const int* slots, const int32_t* counts, in
 
   st_status st = flush_tables(P, s);
   if (st != ST_OK) return poison(P, st);
+  if (deferred && cows.empty()) {
+    drop_plan(P, ps);
+    *deferred = true;
+    return ST_OK;
+  }
   const bool inline_plan = n_br <= kInlineAppendBranches && cows.size() <= (size_t)kInlineCows;
   InlineAppendPlan inl;
   const AppendBranch* d_br = nullptr;
@@ -938,15 +947,16 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
   d.part_bytes = part_rows * (c.head_dim + 1) * 4;
 }
 
-// The call's branches as pool slots: live, non-empty, each listed once.
-st_status decode_slots(st_pool* P, const st_seq* br, int n_br, std::vector<int>* slots) {
+// The call's branches as pool slots: live, each listed once, and (unless the
+// call appends a row to each first) non-empty.
+st_status decode_slots(st_pool* P, const st_seq* br, int n_br, std::vector<int>* slots, bool appends = false) {
   if (n_br < 1 || !br) return fail(P, ST_ERR_INVALID, "need at least one branch");
   if (n_br > P->cfg.max_decode_branches)
     return fail(P, ST_ERR_INVALID, "n_br %d > max_decode_branches %d", n_br, P->cfg.max_decode_branches);
   slots->assign(n_br, 0);
   for (int i = 0; i < n_br; ++i) {
     if (!decode_handle(P, br[i], &(*slots)[i])) return fail(P, ST_ERR_INVALID, "stale or unknown handle");
-    if (P->pool->slot((*slots)[i]).len < 1) return fail(P, ST_ERR_INVALID, "decode over an empty sequence");
+    if (!appends && P->pool->slot((*slots)[i]).len < 1) return fail(P, ST_ERR_INVALID, "decode over an empty sequence");
     for (int j = 0; j < i; ++j)
       if ((*slots)[j] == (*slots)[i]) return fail(P, ST_ERR_INVALID, "sequence listed twice");
   }
@@ -955,24 +965,32 @@ st_status decode_slots(st_pool* P, const st_seq* br, int n_br, std::vector<int>*
 
 }  // namespace
 
-ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const void* q, float* o,
-                                float* lse, void* stream) {
-  NvtxRange range_("st_decode_attn");
-  if (!P) return ST_ERR_INVALID;
-  if (st_status b_ = refuse_if_broken(P)) return b_;
-  if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
-  if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
-    return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
-  std::vector<int>& slots = P->call_slots;
-  st_status vs = decode_slots(P, br, n_br, &slots);
-  if (vs != ST_OK) return vs;
+namespace {
+
+// The decode of st_decode_attn and st_decode_step over validated slots.  With
+// app_k / app_v (a decode step whose append was deferred), the item that
+// reads each branch's last page also writes the step's new row into it.
+st_status decode_impl(st_pool* P, const std::vector<int>& slots, const void* q, float* o, float* lse,
+                      cudaStream_t s, const void* app_k, const void* app_v) {
+  const int n_br = (int)slots.size();
   const st_config& c = P->cfg;
   const int G = c.n_q_heads / c.n_kv_heads;
-  DeviceGuard guard(P->device);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-
   DecodePlan& dp = P->plan;
   plan_decode(P, slots, &dp);
+  if (app_k) {
+    // each branch's last page is its own (a shared partial page would have
+    // been copied), so exactly one single-member item holds it
+    int marked = 0;
+    for (AttnItem& it : dp.items) {
+      if (it.n_members != 1) continue;
+      const SeqSlot& ss = P->pool->slot(slots[dp.members[it.member_base]]);
+      if (it.page_begin + it.n_pages == (int32_t)ss.table.size()) {
+        it.flags |= kItemAppend;
+        ++marked;
+      }
+    }
+    if (marked != n_br) return fail(P, ST_ERR_STATE, "decode step: %d of %d new rows placed", marked, n_br);
+  }
   const std::vector<AttnItem>& items = dp.items;
   const std::vector<int32_t>& members = dp.members;
   const std::vector<int32_t>& n_splits = dp.n_splits;
@@ -1031,6 +1049,10 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
   ap.max_pages = c.max_pages;
   ap.max_splits = c.max_splits;
   ap.hold_loads = (c.flags & ST_FLAG_HOLD_LOADS) ? 1 : 0;
+  ap.app_k = static_cast<const __nv_bfloat16*>(app_k);
+  ap.app_v = static_cast<const __nv_bfloat16*>(app_v);
+  ap.k_pool = P->k_pool;
+  ap.v_pool = P->v_pool;
   // a launch whose pages take less than half of L2 is one agent's step or a
   // few: the next step reads the same pages, so they stay in L2
   ap.keep_l2 = bytes < 0.5 * (double)P->l2_bytes ? 1 : 0;
@@ -1049,7 +1071,8 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     if (e != cudaSuccess) return e;
     aw.item_base = n_narrow + n_wide;
     return launch_decode_pair(P->kmap, P->vmap, aw, ip, n_pair, c.head_dim, s);
-  }, (n_narrow > 0 ? 1 : 0) + (n_wide > 0 ? 1 : 0) + (n_pair > 0 ? 1 : 0), dp.reread_bytes + part_bytes);
+  }, (n_narrow > 0 ? 1 : 0) + (n_wide > 0 ? 1 : 0) + (n_pair > 0 ? 1 : 0),
+                  dp.reread_bytes + part_bytes);
   if (st != ST_OK) {
     if (ps >= 0) retire_plan(P, ps, s);  // its copy may still be in flight
     return st;
@@ -1076,6 +1099,47 @@ ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const vo
     return st;
   }
   return inline_plan ? ST_OK : retire_plan(P, ps, s);
+}
+
+}  // namespace
+
+ST_API st_status st_decode_attn(st_pool* P, const st_seq* br, int n_br, const void* q, float* o,
+                                float* lse, void* stream) {
+  NvtxRange range_("st_decode_attn");
+  if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
+  if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
+  if (!q || !o || !lse || !aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4))
+    return fail(P, ST_ERR_INVALID, "q/o/lse must be aligned device pointers");
+  std::vector<int>& slots = P->call_slots;
+  st_status vs = decode_slots(P, br, n_br, &slots);
+  if (vs != ST_OK) return vs;
+  DeviceGuard guard(P->device);
+  return decode_impl(P, slots, q, o, lse, static_cast<cudaStream_t>(stream), nullptr, nullptr);
+}
+
+ST_API st_status st_decode_step(st_pool* P, const st_seq* br, int n_br, const void* k, const void* v,
+                                const void* q, float* o, float* lse, void* stream) {
+  NvtxRange range_("st_decode_step");
+  if (!P) return ST_ERR_INVALID;
+  if (st_status b_ = refuse_if_broken(P)) return b_;
+  if (P->meta_only) return fail(P, ST_ERR_STATE, "metadata-only pool has no KV storage");
+  if (!k || !v || !q || !o || !lse || !aligned(k, 16) || !aligned(v, 16) || !aligned(q, 16) || !aligned(o, 16) ||
+      !aligned(lse, 4))
+    return fail(P, ST_ERR_INVALID, "k/v/q/o/lse must be aligned device pointers");
+  std::vector<int>& slots = P->call_slots;
+  st_status st = decode_slots(P, br, n_br, &slots, /*appends=*/true);
+  if (st != ST_OK) return st;
+  DeviceGuard guard(P->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  P->call_counts.assign(n_br, 1);
+  bool deferred = false;
+  st = do_append_rows(P, slots.data(), P->call_counts.data(), n_br, k, v, s, &deferred);
+  if (st != ST_OK) return st;
+  // the rows are in the host tables now: a failure from here on leaves the
+  // device behind them
+  st = decode_impl(P, slots, q, o, lse, s, deferred ? k : nullptr, deferred ? v : nullptr);
+  return st == ST_OK ? ST_OK : poison(P, st);
 }
 
 ST_API st_status st_decode_plan(st_pool* P, const st_seq* br, int n_br, int32_t* items, int item_cap,
