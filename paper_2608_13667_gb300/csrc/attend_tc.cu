@@ -195,6 +195,31 @@ __global__ void __launch_bounds__(kThreads, 2)
 
   // ---- loader --------------------------------------------------------------------
   if (warp == kLoadWarp) {
+    if (!kWide && (item.flags & kItemAppend)) {
+      // a decode step: this run's last key is the row the step appends.  The
+      // warp writes this (layer, KV head)'s K and V of it into the pool (16
+      // bytes per lane) before anything else, so the row is stored even if a
+      // wait of this CTA runs out later, and makes the writes visible to the
+      // TMA copy that loads the page.
+      const int last = n_valid_keys - 1;  // key within the run
+      const int blk = p.table[(int64_t)slot * p.max_pages + page_begin + last / kPageTokens];
+      constexpr int kChunks = D / 8;
+      if (lane < 2 * kChunks) {
+        if ((uint64_t)blk >= (uint64_t)p.n_blocks) {
+          atomicCAS(p.status, 0, kDevBadIndex);
+        } else {
+          const bool is_v = lane >= kChunks;
+          const int c = lane % kChunks;
+          const int64_t src = (((int64_t)layer * p.n_rows_q + members[item.member_base]) * p.Hkv + kvh) * D + c * 8;
+          const int64_t dst =
+              ((((int64_t)layer * p.n_blocks + blk) * p.Hkv + kvh) * kPageTokens + last % kPageTokens) * D + c * 8;
+          *reinterpret_cast<uint4*>((is_v ? p.v_pool : p.k_pool) + dst) =
+              *reinterpret_cast<const uint4*>((is_v ? p.app_v : p.app_k) + src);
+          fence_proxy_async_global();
+        }
+      }
+      __syncwarp();
+    }
     if (p.hold_loads) return;  // test hook: nothing arrives, the other roles' waits run out
     if (lane == 0) {
       prefetch_tensormap(&kmap);
@@ -281,29 +306,6 @@ __global__ void __launch_bounds__(kThreads, 2)
           nxt = base_id + 32 + lane < n_pages ? ids[base_id + 32 + lane] : 0;
         }
         const int np = min(C::kPagesPerStage, n_pages - page0);
-        if ((item.flags & kItemAppend) && jk == n_tiles - 1) {
-          // a decode step: this run's last key is the row the step appends.
-          // The warp writes this (layer, KV head)'s K and V of it into the
-          // pool (16 bytes per lane), then makes the writes visible to the
-          // copies below, which load that page.
-          const int last = n_valid_keys - 1 - page0 * kPageTokens;  // key within the stage
-          int blk = __shfl_sync(0xffffffffu, cur, (page0 - base_id + last / kPageTokens) & 31);
-          constexpr int kChunks = D / 8;
-          if (lane < 2 * kChunks) {
-            if ((uint64_t)blk >= (uint64_t)p.n_blocks) {
-              atomicCAS(p.status, 0, kDevBadIndex);
-            } else {
-              const bool is_v = lane >= kChunks;
-              const int c = lane % kChunks;
-              const int64_t src = (((int64_t)layer * p.n_rows_q + members[item.member_base]) * p.Hkv + kvh) * D + c * 8;
-              const int64_t dst =
-                  ((((int64_t)layer * p.n_blocks + blk) * p.Hkv + kvh) * kPageTokens + last % kPageTokens) * D + c * 8;
-              *reinterpret_cast<uint4*>((is_v ? p.v_pool : p.k_pool) + dst) =
-                  *reinterpret_cast<const uint4*>((is_v ? p.app_v : p.app_k) + src);
-              fence_proxy_async_global();
-            }
-          }
-        }
         if (lane == 0) mbar_arrive_expect_tx(&full[s], 2 * np * page_bytes);
         __syncwarp();
         // one copy per lane (lane = 2 D/64 q + (V ? D/64 : 0) + h): a single

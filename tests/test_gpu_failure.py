@@ -71,3 +71,28 @@ def test_merge_wait_runs_out_and_is_reported(stlib, batched):
     kk, vv = run.context(b, 0)
     o_ref, l_ref = A.merge_prefill(qm2[0].cpu(), kk, vv, L0)
     compare(om[0], lm[0], o_ref, l_ref, "merge after timeout")
+
+
+def test_decode_step_stores_its_row_even_when_the_waits_run_out(stlib):
+    """st_decode_step leaves each new row to the decode kernel that reads its
+    page; that kernel stores the row before any wait, so a decode whose waits
+    run out (ST_FLAG_HOLD_LOADS) still leaves the pool holding what the host
+    tables say it holds."""
+    w = Workload(name="hold_step", n_layers=2, n_q_heads=8, n_kv_heads=2, head_dim=128, n_blocks=32, seed=45)
+    pool = stpkg.Pool(n_layers=2, n_q_heads=8, n_kv_heads=2, head_dim=128, n_blocks=32, seed=45,
+                      max_seqs=4, max_decode_branches=2, max_splits=4, flags=stpkg.ST_FLAG_HOLD_LOADS)
+    a, b = pool.seq_create(), pool.seq_create()
+    k, v = kv_rows(w, ("ctx",), 20, device="cuda")
+    pool.append_kv([a, b], k.view(2, 2, 10, 2, 128), v.view(2, 2, 10, 2, 128))
+    kn, vn = kv_rows(w, ("new",), 2, device="cuda")            # [L][2 branches][Hkv][D]
+    pool.decode_step([a, b], kn, vn, queries(w, ("q",), 2, device="cuda"))
+    with pytest.raises(stpkg.STError) as e:
+        pool.sync()
+    assert e.value.status == stpkg.ST_ERR_TIMEOUT
+    for i, h in enumerate((a, b)):
+        table, n = pool.block_table(h)
+        assert n == 11
+        page, row = table[(n - 1) // 16], (n - 1) % 16
+        assert torch.equal(pool.k_pool[:, page, :, row], kn[:, i])
+        assert torch.equal(pool.v_pool[:, page, :, row], vn[:, i])
+    pool.close()
