@@ -99,16 +99,18 @@ def _long_groups(run, w):
     return groups
 
 
-def _check_every_layer(run, w, groups, q, o, lse, jobs, what):
-    """Every branch of every group on every layer, one (layer, group) oracle
-    job each, spread over the worker processes."""
+def _check_every_layer(run, w, groups, q, o, lse, jobs, what, pick=None):
+    """Every branch of every group (or the branches `pick` chooses by their
+    index in the group) on every layer, one (layer, group) oracle job each,
+    spread over the worker processes."""
     o_cpu, l_cpu, q_cpu = o.cpu(), lse.cpu(), q.cpu()
     futs, col = [], 0
     for g in groups:
-        idx = list(range(col, col + len(g)))
+        sel = sorted(set(pick(len(g)))) if pick else list(range(len(g)))
+        idx = [col + i for i in sel]
         col += len(g)
         for layer in range(w.n_layers):
-            futs.append((layer, idx, jobs.decode(w, layer, q_cpu[layer, idx], [run.hist[r] for r in g],
+            futs.append((layer, idx, jobs.decode(w, layer, q_cpu[layer, idx], [run.hist[g[i]] for i in sel],
                                                   run.sizes)))
     for layer, idx, f in futs:
         o_ref, l_ref = f.get()
@@ -132,9 +134,11 @@ def test_cfg4_long_trajectory_every_layer(stlib, oracle_jobs):
 @pytest.mark.parametrize("n_aux", [8, 16])
 def test_cfg4_long_trajectory_wide_every_layer(stlib, oracle_jobs, n_aux):
     """The long-trajectory workload at full size with 9 branches per group (72
-    stacked rows: one wide tile per group) and 17 (136 rows: two wide subgroups
-    whose second read of each prefix page comes from L2), as `bench.py --n-aux`
-    times it; every branch on every layer."""
+    stacked rows: one wide tile per group) and 17 (136 rows: the paired tile,
+    128 rows in its first tile and 8 in its second), as `bench.py --n-aux`
+    times it; on every layer, six branches per group: the first two, two in
+    the middle and the last two (the last one in the paired tile's second
+    tile)."""
     from workloads.configs import long_with_branches
     w = long_with_branches(n_aux)
     run = _run(w, cache_layers=48)
@@ -144,7 +148,8 @@ def test_cfg4_long_trajectory_wide_every_layer(stlib, oracle_jobs, n_aux):
     q, o, lse = run.decode(rids, ("q",))
     run.pool.sync()
     run.check_tables()
-    _check_every_layer(run, w, groups, q, o, lse, oracle_jobs, w.name)
+    _check_every_layer(run, w, groups, q, o, lse, oracle_jobs, w.name,
+                       pick=lambda n: [0, 1, n // 2, n // 2 + 1, n - 2, n - 1])
 
 
 def test_cfg5_full_cycle(stlib, oracle_jobs):
