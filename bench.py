@@ -161,13 +161,21 @@ def _ncu_traffic(kernel, workload):
 
 # --------------------------------------------------------------------------- ours
 
-def build_long_workload(w, dev):
-    """Pool with 4 fork groups at full size; returns (pool, branch handles)."""
+def build_long_workload(w, dev, step_rows=0):
+    """The workload's fork groups at full size in a pool with room for
+    step_rows more rows per branch; returns (pool, branch handles)."""
     import torch
     import paper_2608_13667_gb300 as st
     from workloads import kv_rows
+    n_br = w.n_tasks * (w.n_aux + 1)
+    extra = -(-step_rows // 16) + 1  # pages a branch may take for the steps
+    limits = dict(w.limits)
+    if step_rows:
+        longest = max(p + max(s) for p, s in zip(w.prefix, w.suffix))
+        limits["max_pages"] = max(limits.get("max_pages", 0), -(-longest // 16) + extra)
     pool = st.Pool(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
-                   head_dim=w.head_dim, n_blocks=w.n_blocks, seed=w.seed, device=dev, **w.limits)
+                   head_dim=w.head_dim, n_blocks=w.n_blocks + (n_br * extra if step_rows else 0), seed=w.seed,
+                   device=dev, **limits)
     shape = lambda n: (w.n_layers, 1, n, w.n_kv_heads, w.head_dim)
     branches = []
     for t in range(w.n_tasks):
@@ -219,7 +227,9 @@ def run_ours(args, rank, ws, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     st.build()
-    pool, br = build_long_workload(w, dev)
+    # rows each branch takes: warm-up and timed steps, the end-to-end run (at
+    # most 12) and the latency record's two loops (5 + steps each)
+    pool, br = build_long_workload(w, dev, step_rows=args.warmup + 3 * args.steps + 32)
     n_br = len(br)
     n_steps = args.warmup + args.steps
     # per-step inputs, resident in HBM before the timed region
