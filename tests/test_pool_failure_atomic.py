@@ -82,3 +82,19 @@ def test_ragged_prefill_out_of_pages_changes_nothing(stlib):
     ref.prefill_batch(rs, [12, 20, 80])
     assert lp.free_list() == list(ref.free) == []
     assert [lp.block_table(h)[0] for h in hs] == [ref.seqs[r].table for r in rs]
+
+
+def test_decode_calls_on_a_metadata_pool_change_nothing(stlib):
+    """A metadata-only pool has no KV storage: the attention calls, and the
+    decode step that would append before its decode, are refused with
+    ST_ERR_STATE and leave the tables as they were."""
+    import ctypes
+    lp = _meta(stlib, n_blocks=16, max_seqs=4)
+    a = lp.seq_create()
+    lp.append_kv([a], 5, None)
+    before = _state(lp, [a])
+    L = stlib.lib()
+    arr = (ctypes.c_int64 * 1)(a)
+    assert L.st_decode_step(lp._h, arr, 1, None, None, None, None, None, None) == stlib.ST_ERR_STATE
+    assert L.st_decode_attn(lp._h, arr, 1, None, None, None, None) == stlib.ST_ERR_STATE
+    assert _state(lp, [a]) == before
