@@ -340,7 +340,12 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (lane == 0) {
       constexpr uint32_t idesc_s = tc_idesc_bf16(C::kM, C::kKeys, 0, 0);
       constexpr uint32_t idesc_o = tc_idesc_bf16(C::kM, D, 0, 1);
-      const uint32_t q_addr = smem_addr(q_s);
+      // Shared-memory descriptors are built once: the start field holds
+      // address / 16 (below 2^14 in shared memory), so the descriptor of an
+      // operand shifted by b bytes is the base descriptor + b / 16.
+      const uint64_t q_desc = tc_desc_sw128(smem_addr(q_s), 16, 1024);
+      const uint64_t k_desc0 = tc_desc_sw128(smem_addr(ring), 16, 1024);
+      const uint64_t v_desc0 = tc_desc_sw128(smem_addr(ring + C::kKSlotBytes), C::kKVHalfBytes, 1024);
       bool ok = mbar_wait(q_ready, 0);
       tc_fence_after_sync();
       // S_j = Q K_j^T into S buffer j & 1
@@ -348,15 +353,14 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int s = j % C::kStages;
         if (!mbar_wait(&full[s], (j / C::kStages) & 1)) return false;
         tc_fence_after_sync();
-        const uint32_t k_addr = smem_addr(ring + s * C::kStageBytes);
+        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
 #pragma unroll
         for (int h = 0; h < C::kHalves; ++h)
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
             tc_mma_bf16(tmem + kTmemS + (j & 1) * C::kKeys,
-                        tc_desc_sw128(q_addr + h * C::kQHalfBytes + kk * 32, 16, 1024),
-                        tc_desc_sw128(k_addr + h * C::kKVHalfBytes + kk * 32, 16, 1024), idesc_s,
-                        (h | kk) != 0);
+                        q_desc + (uint64_t)((h * C::kQHalfBytes + kk * 32) >> 4),
+                        kd + (uint64_t)((h * C::kKVHalfBytes + kk * 32) >> 4), idesc_s, (h | kk) != 0);
         tc_commit(&s_full[j & 1]);
         if constexpr (C::kSplitKV) tc_commit(&empty[s]);  // K_j has been read
         return true;
@@ -382,8 +386,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         tc_fence_after_sync();
         const int s = j % C::kStages;
-        const uint32_t k_addr = smem_addr(ring + s * C::kStageBytes);
-        const uint32_t v_addr = k_addr + C::kKSlotBytes;
+        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
+        const uint64_t vd0 = v_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
         if constexpr (kWide) {
           if (!mbar_wait(&v_full[s], (j / C::kStages) & 1)) {
             ok = false;
@@ -394,20 +398,19 @@ __global__ void __launch_bounds__(kThreads, 2)
           const uint32_t p_tm = tmem + kTmemS + (j & 1) * C::kKeys;
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks) {
-            const uint64_t vd = tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024);
+            const uint64_t vd = vd0 + (uint64_t)((ks * 16 * 128) >> 4);
             tc_mma_bf16_tmem_a(tmem + kTmemO, p_tm + ks * 16, vd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
             tc_mma_bf16_tmem_a(tmem + kTmemO, p_tm + ks * 16 + 8, vd, idesc_o, 1u);
           }
         } else {
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks)
-            tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + ks * 32, 16, 1024),
-                        tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o,
-                        (j > 0 || ks > 0) ? 1u : 0u);
+            tc_mma_bf16(tmem + kTmemO, kd + (uint64_t)((ks * 32) >> 4), vd0 + (uint64_t)((ks * 16 * 128) >> 4),
+                        idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks)
-            tc_mma_bf16(tmem + kTmemO, tc_desc_sw128(k_addr + C::kPloOffset + ks * 32, 16, 1024),
-                        tc_desc_sw128(v_addr + ks * 16 * 128, C::kKVHalfBytes, 1024), idesc_o, 1u);
+            tc_mma_bf16(tmem + kTmemO, kd + (uint64_t)((C::kPloOffset + ks * 32) >> 4),
+                        vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o, 1u);
         }
         tc_commit(C::kSplitKV ? &v_empty[s] : &empty[s]);
         tc_commit(o_ready);
