@@ -124,7 +124,7 @@ struct TcCfg {
   static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 };
 
-template <int D, bool kWide>
+template <int D, bool kWide, bool kElect>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
@@ -336,8 +336,30 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 
   // ---- MMA issuer ----------------------------------------------------------------
+  // One lane runs the issue loop; in the kElect form (small launches whose
+  // pages stay in L2, where a step is a chain of latencies) the whole warp
+  // runs it with warp-uniform operands and an elected lane issues, which
+  // shortens each hand-off but costs the streaming launches issue slots.
   if (warp == kMmaWarp) {
-    if (lane == 0) {
+    auto wait = [&](uint64_t* bar, uint32_t parity) {
+      return kElect ? __all_sync(0xffffffffu, mbar_wait(bar, parity)) : mbar_wait(bar, parity);
+    };
+    auto landed = [&](uint64_t* bar, uint32_t parity) {
+      return kElect ? __all_sync(0xffffffffu, mbar_try_wait(bar, parity)) : mbar_try_wait(bar, parity);
+    };
+    auto mma_ss = [&](uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+      if constexpr (kElect) tc_mma_bf16_elect(d, a, b, idesc, acc);
+      else tc_mma_bf16(d, a, b, idesc, acc);
+    };
+    auto mma_ts = [&](uint32_t d, uint32_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+      if constexpr (kElect) tc_mma_bf16_tmem_a_elect(d, a, b, idesc, acc);
+      else tc_mma_bf16_tmem_a(d, a, b, idesc, acc);
+    };
+    auto commit = [&](uint64_t* bar) {
+      if constexpr (kElect) tc_commit_elect(bar);
+      else tc_commit(bar);
+    };
+    if (kElect || lane == 0) {
       constexpr uint32_t idesc_s = tc_idesc_bf16(C::kM, C::kKeys, 0, 0);
       constexpr uint32_t idesc_o = tc_idesc_bf16(C::kM, D, 0, 1);
       // Shared-memory descriptors are built once: the start field holds
@@ -346,23 +368,22 @@ __global__ void __launch_bounds__(kThreads, 2)
       const uint64_t q_desc = tc_desc_sw128(smem_addr(q_s), 16, 1024);
       const uint64_t k_desc0 = tc_desc_sw128(smem_addr(ring), 16, 1024);
       const uint64_t v_desc0 = tc_desc_sw128(smem_addr(ring + C::kKSlotBytes), C::kKVHalfBytes, 1024);
-      bool ok = mbar_wait(q_ready, 0);
+      bool ok = wait(q_ready, 0);
       tc_fence_after_sync();
       // S_j = Q K_j^T into S buffer j & 1
       auto issue_s = [&](int j) -> bool {
         const int s = j % C::kStages;
-        if (!mbar_wait(&full[s], (j / C::kStages) & 1)) return false;
+        if (!wait(&full[s], (j / C::kStages) & 1)) return false;
         tc_fence_after_sync();
         const uint64_t kd = k_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
 #pragma unroll
         for (int h = 0; h < C::kHalves; ++h)
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
-            tc_mma_bf16(tmem + kTmemS + (j & 1) * C::kKeys,
-                        q_desc + (uint64_t)((h * C::kQHalfBytes + kk * 32) >> 4),
-                        kd + (uint64_t)((h * C::kKVHalfBytes + kk * 32) >> 4), idesc_s, (h | kk) != 0);
-        tc_commit(&s_full[j & 1]);
-        if constexpr (C::kSplitKV) tc_commit(&empty[s]);  // K_j has been read
+            mma_ss(tmem + kTmemS + (j & 1) * C::kKeys, q_desc + (uint64_t)((h * C::kQHalfBytes + kk * 32) >> 4),
+                   kd + (uint64_t)((h * C::kKVHalfBytes + kk * 32) >> 4), idesc_s, (h | kk) != 0);
+        commit(&s_full[j & 1]);
+        if constexpr (C::kSplitKV) commit(&empty[s]);  // K_j has been read
         return true;
       };
       if (ok) ok = issue_s(0);
@@ -373,14 +394,14 @@ __global__ void __launch_bounds__(kThreads, 2)
         // delays P_j V_j.
         const int jn = j + 1;
         bool early = false;
-        if (jn < n_tiles && mbar_try_wait(&full[jn % C::kStages], (jn / C::kStages) & 1)) {
+        if (jn < n_tiles && landed(&full[jn % C::kStages], (jn / C::kStages) & 1)) {
           if (!issue_s(jn)) {
             ok = false;
             break;
           }
           early = true;
         }
-        if (!mbar_wait(&p_full[j & 1], (j >> 1) & 1)) {
+        if (!wait(&p_full[j & 1], (j >> 1) & 1)) {
           ok = false;
           break;
         }
@@ -389,7 +410,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint64_t kd = k_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
         const uint64_t vd0 = v_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
         if constexpr (kWide) {
-          if (!mbar_wait(&v_full[s], (j / C::kStages) & 1)) {
+          if (!wait(&v_full[s], (j / C::kStages) & 1)) {
             ok = false;
             break;
           }
@@ -399,28 +420,28 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks) {
             const uint64_t vd = vd0 + (uint64_t)((ks * 16 * 128) >> 4);
-            tc_mma_bf16_tmem_a(tmem + kTmemO, p_tm + ks * 16, vd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
-            tc_mma_bf16_tmem_a(tmem + kTmemO, p_tm + ks * 16 + 8, vd, idesc_o, 1u);
+            mma_ts(tmem + kTmemO, p_tm + ks * 16, vd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
+            mma_ts(tmem + kTmemO, p_tm + ks * 16 + 8, vd, idesc_o, 1u);
           }
         } else {
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks)
-            tc_mma_bf16(tmem + kTmemO, kd + (uint64_t)((ks * 32) >> 4), vd0 + (uint64_t)((ks * 16 * 128) >> 4),
-                        idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
+            mma_ss(tmem + kTmemO, kd + (uint64_t)((ks * 32) >> 4), vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o,
+                   (j > 0 || ks > 0) ? 1u : 0u);
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks)
-            tc_mma_bf16(tmem + kTmemO, kd + (uint64_t)((C::kPloOffset + ks * 32) >> 4),
-                        vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o, 1u);
+            mma_ss(tmem + kTmemO, kd + (uint64_t)((C::kPloOffset + ks * 32) >> 4),
+                   vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o, 1u);
         }
-        tc_commit(C::kSplitKV ? &v_empty[s] : &empty[s]);
-        tc_commit(o_ready);
+        commit(C::kSplitKV ? &v_empty[s] : &empty[s]);
+        commit(o_ready);
         if (jn < n_tiles && !early && !issue_s(jn)) {
           ok = false;
           break;
         }
       }
-      tc_commit(o_final);
-      if (!ok) atomicCAS(p.status, 0, kDevTimeout);
+      commit(o_final);
+      if (!ok && lane == 0) atomicCAS(p.status, 0, kDevTimeout);
     }
     __syncwarp();
     named_barrier_sync(1, n_swt + 32);
@@ -627,7 +648,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   named_barrier_sync(1, n_swt + 32);
 }
 
-template <int D, bool kWide>
+template <int D, bool kWide, bool kElect>
 cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const AttnParams& p,
                         const InlineDecodePlan& inl, int n_ctas, cudaStream_t s) {
   using C = TcCfg<D, kWide>;
@@ -638,23 +659,24 @@ cudaError_t launch_tc_t(const CUtensorMap& km, const CUtensorMap& vm, const Attn
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    e = cudaFuncSetAttribute(attend_tc_kernel<D, kWide>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(attend_tc_kernel<D, kWide, kElect>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::kSmemBytes);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   dim3 grid(n_ctas, p.Hkv, p.L);
-  return launch_chained(attend_tc_kernel<D, kWide>, grid, dim3(kThreads), C::kSmemBytes, s, km, vm, p, inl);
+  return launch_chained(attend_tc_kernel<D, kWide, kElect>, grid, dim3(kThreads), C::kSmemBytes, s, km, vm, p,
+                        inl);
 }
 
 template <int D>
 int decode_ctas_per_sm_t() {
   using C = TcCfg<D, false>;
-  if (cudaFuncSetAttribute(attend_tc_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(attend_tc_kernel<D, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            C::kSmemBytes) != cudaSuccess)
     return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, false>, kThreads, C::kSmemBytes) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_tc_kernel<D, false, false>, kThreads, C::kSmemBytes) !=
       cudaSuccess)
     return 0;
   return n < 2 ? n : 2;  // two CTAs' TMEM (2 x 256 columns) fill an SM
@@ -667,10 +689,18 @@ cudaError_t launch_decode_tc(const CUtensorMap& km, const CUtensorMap& vm, const
   static const InlineDecodePlan kNone{};
   const InlineDecodePlan& ip = inl ? *inl : kNone;
   if (n_items <= 0) return cudaSuccess;
-  if (D == 128)
-    return wide ? launch_tc_t<128, true>(km, vm, p, ip, n_items, s) : launch_tc_t<128, false>(km, vm, p, ip, n_items, s);
-  if (D == 64)
-    return wide ? launch_tc_t<64, true>(km, vm, p, ip, n_items, s) : launch_tc_t<64, false>(km, vm, p, ip, n_items, s);
+  // the narrow tile of a launch whose pages stay in L2 takes the elected issue
+  const bool elect = !wide && p.keep_l2;
+  if (D == 128) {
+    if (wide) return launch_tc_t<128, true, false>(km, vm, p, ip, n_items, s);
+    return elect ? launch_tc_t<128, false, true>(km, vm, p, ip, n_items, s)
+                 : launch_tc_t<128, false, false>(km, vm, p, ip, n_items, s);
+  }
+  if (D == 64) {
+    if (wide) return launch_tc_t<64, true, false>(km, vm, p, ip, n_items, s);
+    return elect ? launch_tc_t<64, false, true>(km, vm, p, ip, n_items, s)
+                 : launch_tc_t<64, false, false>(km, vm, p, ip, n_items, s);
+  }
   return cudaErrorInvalidValue;
 }
 
