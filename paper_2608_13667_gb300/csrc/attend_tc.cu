@@ -11,8 +11,9 @@
 //
 // Two tile shapes (Section 3.2 lets the branch count vary, so the stacked
 // row count n_b G does):
-//   narrow  M = 64, up to 48 rows (the paper's 1 + 4 branches at G <= 9);
-//           P goes to shared memory over the stage's consumed K slot
+//   narrow  S at M = 64, up to 48 rows (the paper's 1 + 4 branches at
+//           G <= 9); P goes to shared memory over the stage's consumed K
+//           slot, its two bf16 terms stacked as the 128 A rows of one P V
 //   wide    M = 128, up to 128 rows; P stays in TMEM over its own scores and
 //           P V reads it from there (no P in shared memory, so two CTAs still
 //           fit an SM).
@@ -20,11 +21,12 @@
 // pages run next to each other, so the second read of a page comes from L2.
 //
 // CTA layout (192 threads, 2 CTAs per SM):
-//   warps 0..3  softmax (only those with rows run).  Narrow: row r sits in
-//               TMEM lane 32 (r / 16) + r % 16, and threads t and t + 16 of a
-//               warp share row t, each with half of the stage's keys and half
-//               of the O columns (16-lane TMEM loads with a column split).
-//               Wide: thread r owns row r = TMEM lane r.  A thread loads its
+//   warps 0..3  softmax (only those with rows run).  Narrow: row r's scores
+//               sit in TMEM lane 32 (r / 16) + r % 16, and threads t and
+//               t + 16 of a warp share row t, each with half of the stage's
+//               keys (16-lane TMEM loads with a column split); thread t owns
+//               the lane of the row's O_hi, thread t + 16 the lane 16 above
+//               it, which holds O_lo.  Wide: thread r owns row r = TMEM lane r.  A thread loads its
 //               part of its Q row into shared memory; per stage it reads its
 //               scores from TMEM, masks keys past the run, keeps a running max
 //               (narrow: combined with its partner by one shuffle) that is
@@ -46,7 +48,7 @@
 //               reads the page (a branch's last page is its own), so no
 //               separate append launch is needed.
 //   warp 5      TMEM owner; lane 0 issues   S = Q K^T  (M, N=64 keys)
-//               and O += P V (M, N=D) and commits them to mbarriers.  S is
+//               and O += P V (M = 128, N=D) and commits them to mbarriers.  S is
 //               double-buffered in TMEM: S_{j+1} is issued before P_j V_j when
 //               its data has landed, so the softmax of stage j+1 overlaps the
 //               tensor work of stage j.
@@ -59,15 +61,17 @@
 // Shared-memory operands use the 128-byte swizzle (8-row x 128-byte atoms):
 //   Q  [D/64][rows][64]       K-major A (SBO 1024)
 //   K  [D/64][keys][64]       K-major B (SBO 1024)
-//   P  [rows][keys]           narrow: K-major A (SBO 1024), written over K: two
-//                             bf16 terms P_hi, P_lo, one after the other
+//   P  [128][keys]            narrow: K-major A (SBO 1024), written over K:
+//                             P_hi of row r at A row 32 (r / 16) + r % 16,
+//                             P_lo 16 rows below it
 //                             wide: in TMEM, the 16 score columns of keys
 //                             [16 k, 16 k + 16) holding P_hi and P_lo of them
 //   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
-// The narrow MMA computes 64 rows and only the first <= 48 Q and P rows are
-// written; rows past them read whatever follows in shared memory and only
-// produce accumulator rows that nobody reads (each output row depends on its
-// own A row only).  V rows of keys that are not valid (past the run,
+// The narrow S MMA computes 64 rows and only the first <= 48 Q rows are
+// written, and P V reads 128 A rows of which only those of real rows are
+// written; the others read whatever is in shared memory and only produce
+// accumulator rows that nobody reads (each output row depends on its own A
+// row only).  V rows of keys that are not valid (past the run,
 // or in pages a short last stage did not load) are zeroed before P V, so
 // stale shared or pool memory cannot turn 0 * x into NaN in a real row.
 #include <math.h>
@@ -99,8 +103,8 @@ struct TcCfg {
   // K and V slots recycle separately (K and V barrier rings); narrow: P goes
   // over K_j, the two are released together after P_j V_j
   static constexpr bool kSplitKV = kWide;
-  // MMA M = 64 for <= 48 stacked rows: accumulator rows sit in TMEM lanes
-  // 0..15 of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
+  // S at M = 64 for <= 48 stacked rows: score rows sit in TMEM lanes 0..15
+  // of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
   // M = 128 for up to 128 rows (row r at lane r)
   static constexpr int kM = kWide ? 128 : 64;
   static constexpr int kRowsPerWarp = kM / 4;
@@ -108,19 +112,21 @@ struct TcCfg {
   static constexpr int kQHalfBytes = kQRows * 128;
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kKVHalfBytes = kKeys * 128;
-  // P as two bf16 terms (P = P_hi + P_lo, two MMAs against the same V): the
+  // P as two bf16 terms (P = P_hi + P_lo, both against the same V): the
   // rounding of a single bf16 P does not average out when a row sees few
-  // keys or its weights are peaked.  Narrow: both terms over the K slot.
-  static constexpr int kPTermBytes = kWide ? 0 : kQRows * 128;    // one term, kQRows rows
-  static constexpr int kPloOffset = kPTermBytes;                  // P_lo after P_hi in the K slot
-  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, 2 * kPTermBytes);
+  // keys or its weights are peaked.  Narrow: the two terms are the A rows of
+  // one M = 128 product O += [P_hi; P_lo] V, written over the K slot --
+  // P_hi of row r at A row 32 (r / 16) + r % 16 (the lane of r's scores),
+  // P_lo at A row 32 (r / 16) + 16 + r % 16, the lanes M = 64 leaves free in
+  // each warp's quarter -- so the accumulator holds O_hi of row r in one lane
+  // and O_lo in the lane 16 above it, summed at the end.
+  static constexpr int kMo = 128;                                  // M of P V
+  static constexpr int kPBytes = kWide ? 0 : kMo * 128;           // the A rows of P V
+  static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, kPBytes);
   static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
   static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
-  // the MMA reads kM rows of each P term from the last K slot: keep that
-  // inside the allocation
-  static constexpr int kOverread = kWide ? 0 : cmax(0, kPloOffset + kM * 128 - kStageBytes);
-  static constexpr int kBarOffset = kQBytes + kRingBytes + kOverread;
+  static constexpr int kBarOffset = kQBytes + kRingBytes;
   static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 };
 
@@ -361,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     };
     if (kElect || lane == 0) {
       constexpr uint32_t idesc_s = tc_idesc_bf16(C::kM, C::kKeys, 0, 0);
-      constexpr uint32_t idesc_o = tc_idesc_bf16(C::kM, D, 0, 1);
+      constexpr uint32_t idesc_o = tc_idesc_bf16(C::kMo, D, 0, 1);
       // Shared-memory descriptors are built once: the start field holds
       // address / 16 (below 2^14 in shared memory), so the descriptor of an
       // operand shifted by b bytes is the base descriptor + b / 16.
@@ -424,14 +430,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             mma_ts(tmem + kTmemO, p_tm + ks * 16 + 8, vd, idesc_o, 1u);
           }
         } else {
+          // [P_hi; P_lo] V: one M = 128 product per 16 keys for both terms
 #pragma unroll
           for (int ks = 0; ks < C::kKeys / 16; ++ks)
             mma_ss(tmem + kTmemO, kd + (uint64_t)((ks * 32) >> 4), vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o,
                    (j > 0 || ks > 0) ? 1u : 0u);
-#pragma unroll
-          for (int ks = 0; ks < C::kKeys / 16; ++ks)
-            mma_ss(tmem + kTmemO, kd + (uint64_t)((C::kPloOffset + ks * 32) >> 4),
-                   vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o, 1u);
         }
         commit(C::kSplitKV ? &v_empty[s] : &empty[s]);
         commit(o_ready);
@@ -452,12 +455,12 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (warp >= n_sw) return;
 
   // ---- softmax warps ---------------------------------------------------------------
-  // Narrow: threads t and t + 16 of a warp share row t, half of the stage's
-  // keys and half of the O columns each, the row max and sum combined with
-  // one shuffle.  Wide: one thread per row.
+  // Narrow: threads t and t + 16 of a warp share row t and half of the
+  // stage's keys each, the row max and sum combined with one shuffle; thread
+  // t owns the TMEM lane of O_hi (P_hi V) of the row, thread t + 16 the lane
+  // of O_lo (P_lo V).  Wide: one thread per row.
   constexpr bool kPair = !kWide;
   constexpr int kKpt = C::kKeys / (kPair ? 2 : 1);  // keys per thread per stage
-  constexpr int kOpt = D / (kPair ? 2 : 1);         // O columns per thread
   const int tid = threadIdx.x;                      // 0 .. n_swt-1, for cooperative loops
   const int half = kPair ? (lane >> 4) : 0;
   const int r = kPair ? warp * 16 + (lane & 15) : threadIdx.x;  // this thread's row
@@ -481,16 +484,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   mbar_arrive(q_ready);
 
-  // this thread's 32-column pieces of its O row: [o_col(k), o_col(k) + 32)
-  auto o_load = [&](int k, float* o) {
-    if constexpr (kPair) tmem_ld16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
-    else tmem_ld32(t_lane + kTmemO + k * 32, o);
-  };
-  auto o_store = [&](int k, const float* o) {
-    if constexpr (kPair) tmem_st16x2_32<D / 2>(t_lane + kTmemO + k * 32, o);
-    else tmem_st32(t_lane + kTmemO + k * 32, o);
-  };
-  auto o_col = [&](int k) { return half * (D / 2) + k * 32; };
+  // columns [32 k, 32 k + 32) of this thread's O lane
+  auto o_load = [&](int k, float* o) { tmem_ld32(t_lane + kTmemO + k * 32, o); };
+  auto o_store = [&](int k, const float* o) { tmem_st32(t_lane + kTmemO + k * 32, o); };
 
   const float sl2 = p.scale_log2;
   float m_used = -1e30f, l = 0.f;  // l: this thread's share of the row sum
@@ -539,7 +535,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         tc_fence_after_sync();
 #pragma unroll 1
-        for (int k = 0; k < kOpt / 32; ++k) {
+        for (int k = 0; k < D / 32; ++k) {
           float o[32];
           o_load(k, o);
 #pragma unroll
@@ -587,12 +583,14 @@ __global__ void __launch_bounds__(kThreads, 2)
         pl[c / 2] = pack_bf16(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
       }
       l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
+      // A rows of P_hi and P_lo: 32 w + t and 32 w + 16 + t (both = t mod 8)
+      const int a_hi = warp * 32 + (lane & 15);
 #pragma unroll
       for (int cc = 0; cc < kKpt / 8; ++cc) {
         const int c = half * (kKpt / 8) + cc;  // 16-byte chunk of the P row (8 keys)
-        const uint32_t off = r * 128 + ((c ^ (r & 7)) << 4);
+        const uint32_t off = a_hi * 128 + ((c ^ (a_hi & 7)) << 4);
         *reinterpret_cast<uint4*>(kslot + off) = make_uint4(pk[4 * cc], pk[4 * cc + 1], pk[4 * cc + 2], pk[4 * cc + 3]);
-        *reinterpret_cast<uint4*>(kslot + C::kPloOffset + off) =
+        *reinterpret_cast<uint4*>(kslot + 16 * 128 + off) =
             make_uint4(pl[4 * cc], pl[4 * cc + 1], pl[4 * cc + 2], pl[4 * cc + 3]);
       }
     }
@@ -629,15 +627,38 @@ __global__ void __launch_bounds__(kThreads, 2)
       dst = p.out_o + idx * D;
       if (half == 0) dst_lse = p.out_lse + idx;
     }
+    if constexpr (kPair) {
+      // O = O_hi + O_lo: thread t writes columns [0, D/2) of the row, thread
+      // t + 16 columns [D/2, D); one shuffle per column pair swaps the halves
+      // each needs from the other's lane
 #pragma unroll 1
-    for (int k = 0; k < kOpt / 32; ++k) {
-      float o[32];
-      o_load(k, o);
-      if (dst) {
+      for (int k = 0; k < D / 64; ++k) {
+        float a[32], b[32];
+        o_load(k, a);           // columns [32 k, 32 k + 32)
+        o_load(k + D / 64, b);  // columns [D/2 + 32 k, D/2 + 32 k + 32)
 #pragma unroll
-        for (int i = 0; i < 32; i += 4)
-          *reinterpret_cast<float4*>(dst + o_col(k) + i) =
-              make_float4(o[i] * inv, o[i + 1] * inv, o[i + 2] * inv, o[i + 3] * inv);
+        for (int i = 0; i < 32; ++i) {
+          const float other = __shfl_xor_sync(0xffffffffu, half ? a[i] : b[i], 16);
+          a[i] = (half ? b[i] : a[i]) + other;
+        }
+        if (dst) {
+          float* d = dst + half * (D / 2) + k * 32;
+#pragma unroll
+          for (int i = 0; i < 32; i += 4)
+            *reinterpret_cast<float4*>(d + i) = make_float4(a[i] * inv, a[i + 1] * inv, a[i + 2] * inv, a[i + 3] * inv);
+        }
+      }
+    } else {
+#pragma unroll 1
+      for (int k = 0; k < D / 32; ++k) {
+        float o[32];
+        o_load(k, o);
+        if (dst) {
+#pragma unroll
+          for (int i = 0; i < 32; i += 4)
+            *reinterpret_cast<float4*>(dst + k * 32 + i) =
+                make_float4(o[i] * inv, o[i + 1] * inv, o[i + 2] * inv, o[i + 3] * inv);
+        }
       }
     }
     if (dst_lse) *dst_lse = (m_used + log2f(l)) * kLn2;
