@@ -6,13 +6,13 @@
 // is dominated by those cached-prefix reads.  A decode CTA owns one run of
 // pages of one KV head of one layer and stacks every query row that reads
 // it -- for a shared prefix all branches of the fork group x the G query
-// heads of the KV head (<= 48 rows) -- so each prefix page crosses HBM once
+// heads of the KV head (<= 64 rows) -- so each prefix page crosses HBM once
 // per group.
 //
 // Two tile shapes (Section 3.2 lets the branch count vary, so the stacked
 // row count n_b G does):
-//   narrow  S at M = 64, up to 48 rows (the paper's 1 + 4 branches at
-//           G <= 9); P goes to shared memory over the stage's consumed K
+//   narrow  S at M = 64, up to 64 rows (the paper's 1 + 4 branches at
+//           G <= 12); P goes to shared memory over the stage's consumed K
 //           slot, its two bf16 terms stacked as the 128 A rows of one P V
 //   wide    M = 128, up to 128 rows; P stays in TMEM over its own scores and
 //           P V reads it from there (no P in shared memory, so two CTAs still
@@ -67,8 +67,7 @@
 //                             wide: in TMEM, the 16 score columns of keys
 //                             [16 k, 16 k + 16) holding P_hi and P_lo of them
 //   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
-// The narrow S MMA computes 64 rows and only the first <= 48 Q rows are
-// written, and P V reads 128 A rows of which only those of real rows are
+// The narrow P V reads 128 A rows of which only those of real rows are
 // written; the others read whatever is in shared memory and only produce
 // accumulator rows that nobody reads (each output row depends on its own A
 // row only).  V rows of keys that are not valid (past the run,
@@ -103,12 +102,12 @@ struct TcCfg {
   // K and V slots recycle separately (K and V barrier rings); narrow: P goes
   // over K_j, the two are released together after P_j V_j
   static constexpr bool kSplitKV = kWide;
-  // S at M = 64 for <= 48 stacked rows: score rows sit in TMEM lanes 0..15
+  // S at M = 64 for <= 64 stacked rows: score rows sit in TMEM lanes 0..15
   // of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
   // M = 128 for up to 128 rows (row r at lane r)
   static constexpr int kM = kWide ? 128 : 64;
   static constexpr int kRowsPerWarp = kM / 4;
-  static constexpr int kQRows = kWide ? 128 : 48;      // Q rows stored
+  static constexpr int kQRows = kWide ? 128 : 64;      // Q rows stored
   static constexpr int kQHalfBytes = kQRows * 128;
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kKVHalfBytes = kKeys * 128;
@@ -127,7 +126,11 @@ struct TcCfg {
   static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
   static constexpr int kBarOffset = kQBytes + kRingBytes;
-  static constexpr int kSmemBytes = 1024 + kBarOffset + 256;
+  // no alignment slack: two narrow CTAs of 64 rows fill an SM's shared
+  // memory, so the kernel requires the dynamic shared memory to start on a
+  // 1024-byte boundary (it does when a kernel has no static shared memory;
+  // the kernel checks and reports ST_ERR_CUDA otherwise)
+  static constexpr int kSmemBytes = kBarOffset + 256;
 };
 
 template <int D, bool kWide, bool kElect>
@@ -135,9 +138,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const AttnParams p, const __grid_constant__ InlineDecodePlan inl) {
   using C = TcCfg<D, kWide>;
-  extern __shared__ uint8_t smem_raw[];
-  const uint32_t raw = smem_addr(smem_raw);
-  uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if (smem_addr(smem_raw) & 1023u) {  // the 128-byte swizzle needs 1024-byte aligned operands
+    griddep_wait();
+    if (threadIdx.x == 0) atomicCAS(p.status, 0, kDevBadSmem);
+    return;
+  }
+  uint8_t* base = smem_raw;
   uint8_t* q_s = base;
   uint8_t* ring = base + C::kQBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::kBarOffset);

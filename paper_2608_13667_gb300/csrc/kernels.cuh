@@ -18,6 +18,7 @@ constexpr int kPageTokens = 16;
 
 // Device status word codes (mirrors st_status values).
 constexpr int32_t kDevBadIndex = 1;
+constexpr int32_t kDevBadSmem = 4;  // dynamic shared memory not where a kernel needs it
 constexpr int32_t kDevTimeout = 5;
 
 struct TableRun {
@@ -69,7 +70,7 @@ struct AttnItem {
 };
 // a sibling item (another subgroup of the fork group) reads the same pages
 constexpr int32_t kItemReread = 1;
-// more than 48 stacked rows: the M = 128 tile
+// more than 64 stacked rows: the M = 128 tile
 constexpr int32_t kItemWide = 2;
 // more than 128 stacked rows: two M = 128 tiles of one CTA sharing every K/V
 // stage (the merge's paired tile, merge_tc.cu)

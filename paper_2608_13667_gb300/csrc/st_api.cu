@@ -34,7 +34,8 @@ namespace {
 
 constexpr int kStageSlots = 8;
 constexpr size_t kStageSlotBytes = 2u << 20;  // 2 MiB per plan
-constexpr int kMaxAttnRows = 48;              // stacked query rows of the narrow decode tile
+constexpr int kMaxAttnRows = 64;              // stacked query rows of the narrow decode tile
+constexpr int kMaxGqa = 48;                   // query heads per KV head
 constexpr int kMaxWideRows = 128;             // ... of the wide one
 constexpr int kMaxPairRows = 256;             // ... and of the paired tile
 
@@ -57,7 +58,7 @@ bool config_valid(const st_config* c, std::string* why) {
   if (c->n_layers < 1) return bad("n_layers must be >= 1");
   if (c->n_kv_heads < 1 || c->n_q_heads < 1 || c->n_q_heads % c->n_kv_heads != 0)
     return bad("n_kv_heads must divide n_q_heads");
-  if (c->n_q_heads / c->n_kv_heads > kMaxAttnRows) return bad("n_q_heads / n_kv_heads must be <= 48");
+  if (c->n_q_heads / c->n_kv_heads > kMaxGqa) return bad("n_q_heads / n_kv_heads must be <= 48");
   if (c->head_dim != 64 && c->head_dim != 128) return bad("head_dim must be 64 or 128");
   if (c->page_size != kPageTokens) return bad("page_size must be 16");
   if (c->max_seqs < 1) return bad("max_seqs must be >= 1");
@@ -742,7 +743,7 @@ namespace {
 // their block tables) are read once for all of them; each branch's own pages
 // are read for it alone.  Runs of pages are sized to the SM count (about 64
 // waves of two CTAs per SM, at least 16 pages), the tile shape follows the
-// stacked rows (narrow up to 48, wide up to 128, paired up to 256, balanced
+// stacked rows (narrow up to 64, wide up to 128, paired up to 256, balanced
 // paired subgroups beyond), and the items come out narrow first, then wide,
 // then paired, longest first within each.
 void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
@@ -775,7 +776,7 @@ void plan_decode(st_pool* P, const std::vector<int>& slots, DecodePlan* out) {
     while (f0 + nm < n_br && d.fam_of[d.by_fam[f0 + nm]] == k) ++nm;
     const int32_t* mem = d.by_fam.data() + f0;
     f0 += nm;
-    // one narrow tile (<= 48 stacked rows), else one wide tile (<= 128), else
+    // one narrow tile (<= 64 stacked rows), else one wide tile (<= 128), else
     // one paired tile (<= 256), else paired subgroups
     const int rows = nm * G;
     const int tile = rows <= kMaxAttnRows ? 0 : rows <= kMaxWideRows ? 1 : 2;
@@ -1372,6 +1373,7 @@ ST_API st_status st_sync(st_pool* P, void* stream) {
   if (code != 0) {
     CUDA_TRY(P, cudaMemset(P->d_status, 0, sizeof code));
     if (code == kDevTimeout) return fail(P, ST_ERR_TIMEOUT, "a device-side wait ran past its limit");
+    if (code == kDevBadSmem) return fail(P, ST_ERR_CUDA, "a kernel's dynamic shared memory was not 1024-byte aligned");
     return fail(P, ST_ERR_INVALID, "a device-side bounds check failed (code %d)", code);
   }
   return ST_OK;

@@ -9,7 +9,7 @@ import pytest
 import paper_2608_13667_gb300 as stpkg
 
 PAGE = 16
-NARROW_ROWS, WIDE_ROWS, PAIR_ROWS = 48, 128, 256
+NARROW_ROWS, WIDE_ROWS, PAIR_ROWS = 64, 128, 256
 WIDE, REREAD, PAIR = 2, 1, 4
 
 
@@ -110,10 +110,11 @@ def test_shared_prefix_is_read_once_per_group(stlib):
     assert all(it["n_members"] == 5 and not it["flags"] & WIDE for it in shared)
 
 
-@pytest.mark.parametrize("n_br,G,tiles", [(6, 8, 1), (16, 8, 1), (17, 8, 1), (40, 4, 1), (9, 16, 1), (32, 8, 1),
-                                         (33, 8, 2), (48, 8, 2), (6, 48, 2), (48, 16, 3)])
+@pytest.mark.parametrize("n_br,G,tiles", [(6, 8, 1), (7, 8, 1), (8, 8, 1), (9, 8, 1), (13, 5, 1), (16, 8, 1),
+                                         (17, 8, 1), (40, 4, 1), (9, 16, 1), (32, 8, 1), (33, 8, 2), (48, 8, 2),
+                                         (6, 48, 2), (48, 16, 3)])
 def test_tile_choice_follows_the_stacked_rows(stlib, n_br, G, tiles):
-    """Up to 48 stacked rows: narrow; up to 128: one wide tile; up to 256: one
+    """Up to 64 stacked rows: narrow; up to 128: one wide tile; up to 256: one
     paired tile; beyond: balanced paired subgroups, each over the family's
     common pages, flagged so the sibling's read of a page comes from L2."""
     P = _pool(G, 1, 32)

@@ -131,14 +131,14 @@ def test_cfg4_long_trajectory_every_layer(stlib, oracle_jobs):
     _check_every_layer(run, w, groups, q, o, lse, oracle_jobs, "cfg4")
 
 
-@pytest.mark.parametrize("n_aux", [8, 16])
+@pytest.mark.parametrize("n_aux", [7, 8, 16])
 def test_cfg4_long_trajectory_wide_every_layer(stlib, oracle_jobs, n_aux):
-    """The long-trajectory workload at full size with 9 branches per group (72
-    stacked rows: one wide tile per group) and 17 (136 rows: the paired tile,
-    128 rows in its first tile and 8 in its second), as `bench.py --n-aux`
-    times it; on every layer, six branches per group: the first two, two in
-    the middle and the last two (the last one in the paired tile's second
-    tile)."""
+    """The long-trajectory workload at full size with 8 branches per group (64
+    stacked rows: a full narrow tile, all four softmax warps), 9 (72 rows: one
+    wide tile per group) and 17 (136 rows: the paired tile, 128 rows in its
+    first tile and 8 in its second), as `bench.py --n-aux` times it; on every
+    layer, six branches per group: the first two, two in the middle and the
+    last two (the last one in the paired tile's second tile)."""
     from workloads.configs import long_with_branches
     w = long_with_branches(n_aux)
     run = _run(w, cache_layers=48)
@@ -234,11 +234,14 @@ def _small(D, Hq, Hkv, n_blocks=512, L=2, seed=11, scale=1.0):
     (128, 8, 8, 7, 777, (1, 2, 3, 0, 16, 17, 31, 100)),      # G = 1, eight branches
     (128, 64, 8, 4, 300, (0, 1, 15, 16, 17)),                # G = 8, 40 stacked rows
     (128, 64, 8, 8, 4100, (3,) * 9),                         # 9 x 8 = 72 rows: one wide tile
-    (128, 16, 1, 3, 2000, (0, 9, 0, 40)),                    # G = 16, 64 rows: wide
+    (128, 16, 1, 3, 2000, (0, 9, 0, 40)),                    # G = 16, 64 rows: a full narrow tile
+    (128, 64, 8, 6, 2222, (0, 3, 17, 0, 1, 2, 40)),          # G = 8, 56 rows: narrow, four softmax warps
+    (128, 40, 8, 12, 1800, (1,) * 13),                       # G = 5, 65 rows: one past narrow, wide
+    (64, 64, 4, 3, 1000, (5, 0, 16, 33)),                    # G = 16, 64 rows, D 64: narrow
     (64, 48, 4, 7, 900, (2,) * 8),                           # G = 12, 96 rows: wide, D 64
     (128, 32, 1, 3, 1500, (0, 5, 9, 33)),                    # G = 32, 128 rows: a full wide tile
     (128, 48, 1, 4, 700, (1, 2, 3, 4, 5)),                   # G = 48, 240 rows: wide subgroups 1 + 2 + 2
-    (64, 20, 2, 5, 3333, (0, 7, 16, 31, 64, 65)),            # G = 10, 60 rows: wide, D 64
+    (64, 20, 2, 5, 3333, (0, 7, 16, 31, 64, 65)),            # G = 10, 60 rows: narrow, D 64
     (128, 32, 1, 1, 100, (0, 0)),                            # G = 32, no suffixes
     (64, 4, 1, 0, 50, (0,)),                                 # a lone main thread
     (64, 12, 3, 2, 16, (0, 1, 2)),                           # one-page prefix
