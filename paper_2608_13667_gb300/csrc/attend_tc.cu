@@ -38,9 +38,10 @@
 //               ahead), one 2 KiB TMA copy per (page, 64-wide half of D, K|V)
 //               into a ring of stages, per-stage mbarriers with byte counts;
 //               a stage's copies are issued by the warp's lanes together.
-//               Narrow: one ring, a stage's K and V slots freed together after
-//               its P V.  Wide: K and V have their own barriers; a K slot is
-//               freed by the commit after S_j, a V slot after P_j V_j.
+//               Narrow: one ring of three stages, a stage's K and V slots
+//               freed together after its P V.  Wide: K and V have their own
+//               rings and barriers; a K slot (two of them) is freed by the
+//               commit after S_j, a V slot (three) after P_j V_j.
 //               A decode step (st_decode_step): the narrow item that holds a
 //               branch's last page first stores the step's new K and V row of
 //               its (layer, KV head) into that page, then a proxy fence makes
@@ -97,10 +98,12 @@ struct TcCfg {
   static constexpr int kHalves = D / 64;
   static constexpr int kKeys = 64;                     // keys per stage
   static constexpr int kPagesPerStage = kKeys / kPageTokens;
-  static constexpr int kStages = kWide ? 2 : 3;
   // Wide: P lives in TMEM, so a K slot is free once S_j has been computed and
-  // K and V slots recycle separately (K and V barrier rings); narrow: P goes
-  // over K_j, the two are released together after P_j V_j
+  // K and V slots recycle separately (K and V barrier rings); a V slot is
+  // held until P_j V_j, so V gets the deeper ring.  Narrow: P goes over K_j,
+  // the two are released together after P_j V_j (one ring of stages).
+  static constexpr int kStages = kWide ? 2 : 3;         // K slots
+  static constexpr int kVStages = kWide ? 3 : kStages;  // V slots
   static constexpr bool kSplitKV = kWide;
   // S at M = 64 for <= 64 stacked rows: score rows sit in TMEM lanes 0..15
   // of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
@@ -123,8 +126,9 @@ struct TcCfg {
   static constexpr int kPBytes = kWide ? 0 : kMo * 128;           // the A rows of P V
   static constexpr int kKSlotBytes = cmax(kHalves * kKVHalfBytes, kPBytes);
   static constexpr int kVSlotBytes = kHalves * kKVHalfBytes;
-  static constexpr int kStageBytes = kKSlotBytes + kVSlotBytes;
-  static constexpr int kRingBytes = kStages * kStageBytes;
+  // the K slots, then the V slots
+  static constexpr int kKRingBytes = kStages * kKSlotBytes;
+  static constexpr int kRingBytes = kKRingBytes + kVStages * kVSlotBytes;
   static constexpr int kBarOffset = kQBytes + kRingBytes;
   // no alignment slack: two narrow CTAs of 64 rows fill an SM's shared
   // memory, so the kernel requires the dynamic shared memory to start on a
@@ -150,14 +154,17 @@ __global__ void __launch_bounds__(kThreads, 2)
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::kBarOffset);
   uint64_t* full = bars;                 // [kStages] K (and, narrow, V) landed
   uint64_t* empty = bars + C::kStages;   // [kStages] K (and, narrow, V) slot free
+  // K slot s and V slot s (narrow: the K and V of stage s)
+  auto k_slot = [&](int s) { return ring + s * C::kKSlotBytes; };
+  auto v_slot = [&](int s) { return ring + C::kKRingBytes + s * C::kVSlotBytes; };
   uint64_t* s_full = bars + 2 * C::kStages;   // [2] per S buffer
   uint64_t* p_full = s_full + 2;              // [2] per S buffer
   uint64_t* o_ready = s_full + 4;             // one phase per P V
   uint64_t* o_final = s_full + 5;
   uint64_t* q_ready = s_full + 6;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 7);
-  uint64_t* v_full = s_full + 8;               // [kStages] wide: V landed
-  uint64_t* v_empty = v_full + C::kStages;     // [kStages] wide: V slot free
+  uint64_t* v_full = s_full + 8;               // [kVStages] wide: V landed
+  uint64_t* v_empty = v_full + C::kVStages;    // [kVStages] wide: V slot free
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -187,7 +194,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
-      if (C::kSplitKV) {
+    }
+    if (C::kSplitKV) {
+      for (int s = 0; s < C::kVStages; ++s) {
         mbar_init(&v_full[s], 1);
         mbar_init(&v_empty[s], 1);
       }
@@ -247,10 +256,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     int base_id = 0;
     int cur = lane < n_pages ? ids[lane] : 0;
     int nxt = 32 + lane < n_pages ? ids[32 + lane] : 0;
-    // waits for slot s of a ring to be released for stage j (lane 0 waits)
-    auto slot_free = [&](uint64_t* ring_empty, int s, int j) -> bool {
+    // waits for the slot of stage j in a ring of `depth` slots to be
+    // released (lane 0 waits)
+    auto slot_free = [&](uint64_t* ring_empty, int depth, int j) -> bool {
       int w = 1;
-      if (j >= C::kStages && lane == 0) w = mbar_wait(&ring_empty[s], ((j / C::kStages) - 1) & 1) ? 1 : 0;
+      if (j >= depth && lane == 0) w = mbar_wait(&ring_empty[j % depth], ((j / depth) - 1) & 1) ? 1 : 0;
       return __shfl_sync(0xffffffffu, w, 0) != 0;
     };
     // pages of stage j (j increasing): the count and the TMA page coordinates
@@ -291,27 +301,28 @@ __global__ void __launch_bounds__(kThreads, 2)
     bool ok = true;
     for (; jk < n_tiles; ++jk) {
       const int s = jk % C::kStages;
-      if (!slot_free(empty, s, jk)) {
+      if (!slot_free(empty, C::kStages, jk)) {
         ok = false;
         break;
       }
-      uint8_t* kst = ring + s * C::kStageBytes;
-      uint8_t* vst = kst + C::kKSlotBytes;
+      uint8_t* kst = k_slot(s);
       if constexpr (C::kSplitKV) {
         int c3[C::kPagesPerStage];
         const int np = stage_pages(jk, c3);
         if (lane == 0) mbar_arrive_expect_tx(&full[s], np * page_bytes);
         issue(&kmap, kst, &full[s], c3, np);
-        // the K slot was released by S_j-kStages, the V slot waits for P_j-kStages V_j-kStages
-        if (!slot_free(v_empty, s, jk)) {
+        // the K slot was released by S_j-kStages, the V slot waits for P_j-kVStages V_j-kVStages
+        const int sv = jk % C::kVStages;
+        if (!slot_free(v_empty, C::kVStages, jk)) {
           ok = false;
           ++jk;  // K_j is in flight
           break;
         }
-        if (lane == 0) mbar_arrive_expect_tx(&v_full[s], np * page_bytes);
-        issue(&vmap, vst, &v_full[s], c3, np);
+        if (lane == 0) mbar_arrive_expect_tx(&v_full[sv], np * page_bytes);
+        issue(&vmap, v_slot(sv), &v_full[sv], c3, np);
         jv = jk + 1;
       } else {
+        uint8_t* vst = v_slot(s);
         const int page0 = jk * C::kPagesPerStage;
         if (page0 >= base_id + 32) {
           base_id += 32;
@@ -343,7 +354,8 @@ __global__ void __launch_bounds__(kThreads, 2)
       // wait (bounded) for this CTA's copies still in flight before it exits
       for (int t = max(0, jk - C::kStages); t < jk; ++t) mbar_wait(&full[t % C::kStages], (t / C::kStages) & 1);
       if constexpr (C::kSplitKV)
-        for (int t = max(0, jv - C::kStages); t < jv; ++t) mbar_wait(&v_full[t % C::kStages], (t / C::kStages) & 1);
+        for (int t = max(0, jv - C::kVStages); t < jv; ++t)
+          mbar_wait(&v_full[t % C::kVStages], (t / C::kVStages) & 1);
     }
     return;
   }
@@ -380,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       // operand shifted by b bytes is the base descriptor + b / 16.
       const uint64_t q_desc = tc_desc_sw128(smem_addr(q_s), 16, 1024);
       const uint64_t k_desc0 = tc_desc_sw128(smem_addr(ring), 16, 1024);
-      const uint64_t v_desc0 = tc_desc_sw128(smem_addr(ring + C::kKSlotBytes), C::kKVHalfBytes, 1024);
+      const uint64_t v_desc0 = tc_desc_sw128(smem_addr(ring + C::kKRingBytes), C::kKVHalfBytes, 1024);
       bool ok = wait(q_ready, 0);
       tc_fence_after_sync();
       // S_j = Q K_j^T into S buffer j & 1
@@ -388,7 +400,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int s = j % C::kStages;
         if (!wait(&full[s], (j / C::kStages) & 1)) return false;
         tc_fence_after_sync();
-        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
+        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kKSlotBytes) >> 4);
 #pragma unroll
         for (int h = 0; h < C::kHalves; ++h)
 #pragma unroll
@@ -419,11 +431,11 @@ __global__ void __launch_bounds__(kThreads, 2)
           break;
         }
         tc_fence_after_sync();
-        const int s = j % C::kStages;
-        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
-        const uint64_t vd0 = v_desc0 + (uint64_t)((s * C::kStageBytes) >> 4);
+        const int s = j % C::kStages, sv = j % C::kVStages;
+        const uint64_t kd = k_desc0 + (uint64_t)((s * C::kKSlotBytes) >> 4);
+        const uint64_t vd0 = v_desc0 + (uint64_t)((sv * C::kVSlotBytes) >> 4);
         if constexpr (kWide) {
-          if (!wait(&v_full[s], (j / C::kStages) & 1)) {
+          if (!wait(&v_full[sv], (j / C::kVStages) & 1)) {
             ok = false;
             break;
           }
@@ -443,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             mma_ss(tmem + kTmemO, kd + (uint64_t)((ks * 32) >> 4), vd0 + (uint64_t)((ks * 16 * 128) >> 4), idesc_o,
                    (j > 0 || ks > 0) ? 1u : 0u);
         }
-        commit(C::kSplitKV ? &v_empty[s] : &empty[s]);
+        commit(C::kSplitKV ? &v_empty[sv] : &empty[s]);
         commit(o_ready);
         if (jn < n_tiles && !early && !issue_s(jn)) {
           ok = false;
@@ -553,7 +565,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       l *= alpha;
       if (need) m_used = m_new;
     }
-    uint8_t* kslot = ring + s * C::kStageBytes;  // narrow: S_j has been consumed, P_j goes over K_j
+    uint8_t* kslot = k_slot(s);  // narrow: S_j has been consumed, P_j goes over K_j
     if constexpr (kWide) {
       // P_hi, P_lo of keys [16 k, 16 k + 16) over the 16 TMEM columns of their
       // scores (all read above).  The store is warp-wide: rows past the
@@ -604,11 +616,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (key0 + C::kKeys > n_valid_keys || loaded < C::kKeys) {
       // zero the V rows of keys that are not valid, once V_j has landed
       // (narrow: with K_j, from which S_j was computed)
-      if (!__all_sync(0xffffffffu, mbar_wait(C::kSplitKV ? &v_full[s] : &full[s], (j / C::kStages) & 1))) {
+      const int sv = j % C::kVStages;
+      if (!__all_sync(0xffffffffu, C::kSplitKV ? mbar_wait(&v_full[sv], (j / C::kVStages) & 1)
+                                               : mbar_wait(&full[s], (j / C::kStages) & 1))) {
         ok = false;
         break;
       }
-      uint8_t* vslot = kslot + C::kKSlotBytes;
+      uint8_t* vslot = v_slot(sv);
       for (int t = tid; t < C::kKeys * C::kHalves; t += n_swt) {
         const int c = t % C::kKeys, h = t / C::kKeys;
         if (c >= loaded || key0 + c >= n_valid_keys) {
