@@ -40,8 +40,8 @@
 //               a stage's copies are issued by the warp's lanes together.
 //               Narrow: one ring of three stages, a stage's K and V slots
 //               freed together after its P V.  Wide: K and V have their own
-//               rings and barriers; a K slot (two of them) is freed by the
-//               commit after S_j, a V slot (three) after P_j V_j.
+//               rings of two slots and barriers; a K slot is freed by the
+//               commit after S_j, a V slot after P_j V_j.
 //               A decode step (st_decode_step): the narrow item that holds a
 //               branch's last page first stores the step's new K and V row of
 //               its (layer, KV head) into that page, then a proxy fence makes
@@ -99,11 +99,11 @@ struct TcCfg {
   static constexpr int kKeys = 64;                     // keys per stage
   static constexpr int kPagesPerStage = kKeys / kPageTokens;
   // Wide: P lives in TMEM, so a K slot is free once S_j has been computed and
-  // K and V slots recycle separately (K and V barrier rings); a V slot is
-  // held until P_j V_j, so V gets the deeper ring.  Narrow: P goes over K_j,
-  // the two are released together after P_j V_j (one ring of stages).
+  // K and V slots recycle separately (K and V barrier rings).  Narrow: P goes
+  // over K_j, the two are released together after P_j V_j (one ring of
+  // stages).
   static constexpr int kStages = kWide ? 2 : 3;         // K slots
-  static constexpr int kVStages = kWide ? 3 : kStages;  // V slots
+  static constexpr int kVStages = kWide ? 2 : kStages;  // V slots
   static constexpr bool kSplitKV = kWide;
   // S at M = 64 for <= 64 stacked rows: score rows sit in TMEM lanes 0..15
   // of each warp's 32-lane quarter (row r at lane 32 (r / 16) + r % 16);
