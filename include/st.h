@@ -191,9 +191,10 @@ ST_API st_status st_decode_step(st_pool* pool, const st_seq* br, int n_br, const
  *           whose query rows are stacked on it, split the partial slot it
  *           writes for each of them; flags bit 0: a sibling item of the same
  *           fork family reads the same pages (kept in L2), bit 1: the wide
- *           (M = 128) tile, bit 2: the paired tile (two M = 128 tiles of one
- *           CTA, for 129 to 256 stacked rows).  Narrow items come first, then
- *           wide, then paired.
+ *           (M = 128) tile, for 65 to 128 stacked rows, bit 2: the paired
+ *           tile (two M = 128 tiles of one CTA, for 129 to 256 stacked rows);
+ *           neither: the narrow tile, up to 64 stacked rows.  Narrow items
+ *           come first, then wide, then paired.
  * members:  int32 [member_cap]
  * n_splits: int32 [n_br], partial results per branch (each split index
  *           0 .. n_splits - 1 is written by exactly one item)
