@@ -174,7 +174,7 @@ def compare(o_gpu, lse_gpu, o_ref, lse_ref, what=""):
       with |oracle| >= REL_FLOOR (below it a relative error measures nothing
       but the rounding of a value near zero);
     * the allclose reading, |gpu - oracle| <= 2e-3 + 1e-2 |oracle| per
-      element (implied by the first, kept as the survey states it);
+      element (implied by the first; the per-element form of the same bound);
     and |LSE gpu - LSE oracle| <= 1e-4.  Returns (max_abs, max_rel, max_lse)."""
     o = o_gpu.double().cpu().numpy() if isinstance(o_gpu, torch.Tensor) else np.asarray(o_gpu, np.float64)
     l = lse_gpu.double().cpu().numpy() if isinstance(lse_gpu, torch.Tensor) else np.asarray(lse_gpu, np.float64)
