@@ -332,7 +332,7 @@ ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, in
  *              value covers only what the host can see when the call returns.
  * Branches whose tables start on the same physical page are treated as one
  * fork group: their common full pages are read once for the group (groups
- * of more than 48 / G branches are split into several).
+ * of more than 64 / G branches are split into several).
  * Returns ST_ERR_INVALID for bad arguments or n_br > ST_NOALLOC_MAX_BRANCHES,
  * and ST_ERR_OOM when the call needs more than the static scratch:
  *   36.25 KiB of plan + 4*n_br*table_stride (rounded up to 256 bytes)

@@ -37,7 +37,8 @@ constexpr size_t kScratchBytes = ST_NOALLOC_SCRATCH_BYTES;
 constexpr int kMaxBranches = ST_NOALLOC_MAX_BRANCHES;
 constexpr int kMaxItems = 1024;
 constexpr int kSplitStride = 16;  // partial slots per (layer, branch, head)
-constexpr int kMaxRows = 48;      // stacked query rows per CTA
+constexpr int kMaxRows = 64;      // stacked query rows per CTA (the narrow tile)
+constexpr int kMaxGqa = 48;       // query heads per KV head, as for a pool
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
@@ -122,7 +123,7 @@ extern "C" ST_API st_status st_decode_attn_noalloc(const st_config* geom, const 
     return ST_ERR_INVALID;
   const st_config& c = *geom;
   if (c.n_layers < 1 || c.n_kv_heads < 1 || c.n_q_heads % c.n_kv_heads != 0 ||
-      c.n_q_heads / c.n_kv_heads > kMaxRows || (c.head_dim != 64 && c.head_dim != 128) ||
+      c.n_q_heads / c.n_kv_heads > kMaxGqa || (c.head_dim != 64 && c.head_dim != 128) ||
       c.page_size != kPageTokens || c.n_blocks < 1 || (int64_t)c.n_layers * c.n_blocks >= INT32_MAX)
     return ST_ERR_INVALID;
   if (n_br < 1 || n_br > kMaxBranches || table_stride < 1) return ST_ERR_INVALID;

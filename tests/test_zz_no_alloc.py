@@ -85,8 +85,9 @@ def _two_groups_and_loners():
 
 
 def _family_split():
-    """G = 8: a family of 9 branches exceeds 48 / G = 6 per group and is
-    split; one more sequence is shorter than a page."""
+    """G = 8: a family of 9 branches exceeds 64 / G = 8 per group and is
+    split (a group of 8, and one branch that reads its pages on its own);
+    one more sequence is shorter than a page."""
     w = Workload(name="noalloc_split", n_layers=2, n_q_heads=64, n_kv_heads=8, head_dim=128,
                  n_blocks=1024, seed=24)
     run = Run(w, max_seqs=16, max_decode_branches=16, max_splits=16)
