@@ -272,7 +272,8 @@ ST_API st_status st_free_list(st_pool* pool, int32_t* out, int64_t cap, int64_t*
 
 /* Wait for the stream and report device-side errors raised since the last
  * st_sync (ST_ERR_TIMEOUT for a wait that ran out, ST_ERR_INVALID for a
- * failed bounds check); the device status word is then cleared. */
+ * failed bounds check, ST_ERR_CUDA for a kernel whose dynamic shared memory
+ * was not 1024-byte aligned); the device status word is then cleared. */
 ST_API st_status st_sync(st_pool* pool, void* stream);
 
 /* Kernel accounting.  Launch counts are always kept; with timing enabled
