@@ -328,8 +328,10 @@ ST_API st_status st_profile_read(st_pool* pool, st_kernel_stat* out, int cap, in
  * status:      DEVICE int32 [1], caller-owned.  The call clears it on
  *              `stream` before its kernels run; once the stream has passed
  *              the call it holds ST_OK, ST_ERR_TIMEOUT (a device-side wait ran
- *              past its limit: o and lse are then undefined) or
- *              ST_ERR_INVALID (a device-side bounds check fired).  The return
+ *              past its limit: o and lse are then undefined),
+ *              ST_ERR_INVALID (a device-side bounds check fired) or
+ *              ST_ERR_CUDA (the kernel's dynamic shared memory was not
+ *              1024-byte aligned; nothing computed).  The return
  *              value covers only what the host can see when the call returns.
  * Branches whose tables start on the same physical page are treated as one
  * fork group: their common full pages are read once for the group (groups
