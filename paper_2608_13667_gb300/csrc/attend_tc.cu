@@ -17,17 +17,20 @@
 //   wide    M = 128, up to 128 rows; P stays in TMEM over its own scores and
 //           P V reads it from there (no P in shared memory, so two CTAs still
 //           fit an SM).
-// A group beyond 128 rows is split into subgroups whose items over the same
-// pages run next to each other, so the second read of a page comes from L2.
+// A group of 129 to 256 rows runs on the merge kernel's paired tile
+// (merge_tc.cu); a larger one is split into paired subgroups whose items over
+// the same pages run next to each other, so the second read of a page comes
+// from L2.
 //
 // CTA layout (192 threads, 2 CTAs per SM):
 //   warps 0..3  softmax (only those with rows run).  Narrow: row r's scores
 //               sit in TMEM lane 32 (r / 16) + r % 16, and threads t and
 //               t + 16 of a warp share row t, each with half of the stage's
 //               keys (16-lane TMEM loads with a column split); thread t owns
-//               the lane of the row's O_hi, thread t + 16 the lane 16 above
-//               it, which holds O_lo.  Wide: thread r owns row r = TMEM lane r.  A thread loads its
-//               part of its Q row into shared memory; per stage it reads its
+//               the lane of the row's O_hi, thread t + 16 the lane 16 higher,
+//               which holds O_lo.  Wide: thread r owns row r = TMEM lane r.
+//               A thread loads its part of its Q row into shared memory;
+//               per stage it reads its
 //               scores from TMEM, masks keys past the run, keeps a running max
 //               (narrow: combined with its partner by one shuffle) that is
 //               raised only when a score exceeds it by more than 2^8 (O in
@@ -64,7 +67,7 @@
 //   K  [D/64][keys][64]       K-major B (SBO 1024)
 //   P  [128][keys]            narrow: K-major A (SBO 1024), written over K:
 //                             P_hi of row r at A row 32 (r / 16) + r % 16,
-//                             P_lo 16 rows below it
+//                             P_lo at the A row 16 higher
 //                             wide: in TMEM, the 16 score columns of keys
 //                             [16 k, 16 k + 16) holding P_hi and P_lo of them
 //   V  [D/64][keys][64]       MN-major B (LBO = one D-half, SBO 1024)
